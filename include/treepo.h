@@ -1,0 +1,239 @@
+/*
+ * treepo.h -- C ABI of libtreepo: decode attention over a segment tree of
+ * KV caches on one GB300 (sm_103a).
+ *
+ * TreePO samples each prompt as a tree (Sec. 2.2, Algorithm 1): the prompt is
+ * the root at depth 0, each inference step appends a segment of at most l
+ * tokens to every live path, branching forks a path into b copies, and early
+ * stop drops a path. A trajectory is the concatenation s_1 (+) ... (+) s_j of
+ * the segments on its root-to-leaf path (Sec. 2.3). Sibling branches share
+ * their prefix, which this library stores once (Sec. 2.1: shared prefixes
+ * represented only once; Sec. 1: paths with separate KV caches fail to share)
+ * and reads from HBM once per decode call, not once per branch.
+ *
+ * Objects. One tp_tree owns a paged KV pool and a forest of trees (one root
+ * per prompt). Nodes are dense int32 ids handed out in creation order and
+ * never reused while the tp_tree lives. A node is a live leaf, a frozen
+ * interior node (it has been forked), or dead (pruned).
+ *
+ * Pool. pool_blocks blocks of block_tokens token slots; a block holds K and V
+ * of every kv head for its tokens. An append first fills the node's partly
+ * used last block, then takes new blocks, lowest free index first. Forks move
+ * no bytes: children start empty and read the parent's blocks through the
+ * tree. Token t of a node sits in slot  block[t / block_tokens] * block_tokens
+ * + t % block_tokens.
+ *
+ * Threading and streams. Calls on one tp_tree must not run concurrently. Host
+ * work (validation, tree updates, scheduling) is synchronous; device work is
+ * enqueued on the tree's stream and is asynchronous to the host.
+ *
+ * Errors. Every call returns a tp_status; on failure nothing in the tree
+ * changes and tp_last_error() describes the failure. Kernels never trap: a
+ * bounded wait that runs out sets a device flag that tp_sync() reports as
+ * TP_ERR_DEVICE.
+ *
+ * Pointer conventions. "device" = CUDA device memory (any allocator); "host"
+ * = ordinary host memory. The caller owns every buffer it passes; the library
+ * keeps no pointer to a caller buffer after a call returns, except the pool
+ * arena, which must outlive the tp_tree.
+ */
+#ifndef TREEPO_H_
+#define TREEPO_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t tp_status;
+#define TP_OK 0
+#define TP_ERR_INVALID_ARG (-1) /* bad size, null or misaligned pointer, bad config */
+#define TP_ERR_OOM (-2)         /* pool (or library scratch) exhausted            */
+#define TP_ERR_BAD_NODE (-3)    /* unknown or pruned node id                       */
+#define TP_ERR_FROZEN (-4)      /* append to a node that has been forked           */
+#define TP_ERR_NOT_LEAF (-5)    /* decode/prune of an interior node                */
+#define TP_ERR_EMPTY_PATH (-6)  /* decode of a leaf whose path holds no token      */
+#define TP_ERR_CUDA (-7)        /* a CUDA runtime call failed                      */
+#define TP_ERR_DEVICE (-8)      /* a kernel's bounded wait ran out (tp_sync)       */
+
+typedef int32_t tp_node;
+typedef struct tp_tree tp_tree;
+
+/*
+ * Tree configuration.
+ *   num_q_heads, num_kv_heads: num_q_heads % num_kv_heads == 0; q-head h reads
+ *       kv head h / (num_q_heads / num_kv_heads) (contiguous GQA groups).
+ *   head_dim: 64 or 128.
+ *   block_tokens: tokens per pool block; 32.
+ *   pool_blocks: 1 .. 2^24 blocks.
+ *   pool: device arena of tp_pool_bytes(cfg) bytes, 256-byte aligned, owned
+ *       by the caller and alive as long as the tree; its contents are the
+ *       library's. NULL makes a metadata-only tree: every host operation
+ *       works (append then takes K = V = NULL and copies nothing), device
+ *       operations return TP_ERR_INVALID_ARG. Used to test the host logic
+ *       without a GPU.
+ *   cuda_stream: cudaStream_t for all device work; NULL = legacy default.
+ */
+typedef struct {
+    int32_t num_q_heads;
+    int32_t num_kv_heads;
+    int32_t head_dim;
+    int32_t block_tokens;
+    int64_t pool_blocks;
+    void* pool;
+    void* cuda_stream;
+} tp_config;
+
+/* Bytes the pool arena must hold: pool_blocks * 2 * num_kv_heads *
+ * block_tokens * head_dim * 2 (bf16 K and V). Returns -1 on a bad config. */
+int64_t tp_pool_bytes(const tp_config* cfg);
+
+/* Create an empty forest over cfg's pool. *out receives the handle. */
+tp_status tp_tree_create(const tp_config* cfg, tp_tree** out);
+
+/* Destroy the forest; waits for its device work first. NULL is a no-op. */
+tp_status tp_tree_destroy(tp_tree* tree);
+
+/* Use another stream for subsequent device work (cudaStream_t; NULL = default). */
+tp_status tp_set_stream(tp_tree* tree, void* cuda_stream);
+
+/* New tree: an empty root node (a prompt at depth 0, Sec. 2.2). */
+tp_status tp_add_root(tp_tree* tree, tp_node* out_root);
+
+/*
+ * Append n_tokens tokens to live leaf `node` (a prompt, or a generated
+ * segment s_j: Algorithm 1 concatenates p (+) s). K and V are device bf16
+ * [n_tokens][num_kv_heads][head_dim], 16-byte aligned, already position
+ * encoded; they are copied into pool blocks on the tree's stream (the caller
+ * may reuse them once that stream passes this point). n_tokens == 0 is a
+ * no-op. Errors: TP_ERR_BAD_NODE, TP_ERR_FROZEN (node was forked),
+ * TP_ERR_OOM (not enough free blocks; nothing is allocated),
+ * TP_ERR_INVALID_ARG.
+ */
+tp_status tp_append_segment(tp_tree* tree, tp_node node, int32_t n_tokens, const void* K,
+                            const void* V);
+
+/*
+ * Fork `node` into k >= 1 new empty children (branching, Sec. 2.2: a prompt
+ * forked b times before the next segment). No KV bytes move: the children
+ * read the node's blocks through the tree. The node is frozen (no further
+ * appends); forking a frozen node adds children. out_children: host
+ * array of k ids. Errors: TP_ERR_BAD_NODE, TP_ERR_INVALID_ARG.
+ */
+tp_status tp_fork(tp_tree* tree, tp_node node, int32_t k, tp_node* out_children);
+
+/*
+ * Early stop (Sec. 2.2, heuristic sampling): remove live leaf `leaf`, free
+ * its blocks, and free every ancestor whose last live child it was (a tree
+ * whose leaves are all pruned disappears, root included). Errors:
+ * TP_ERR_BAD_NODE, TP_ERR_NOT_LEAF.
+ */
+tp_status tp_prune(tp_tree* tree, tp_node leaf);
+
+/*
+ * Decode attention for n leaf queries. Row i of Q (device bf16
+ * [n][num_q_heads][head_dim]) attends over every token on the root-to-leaf
+ * path of leaves[i] (host array; a leaf may appear more than once, each
+ * occurrence is its own row). Per q-head h (kv head c):
+ *   s_j = q_h . k_{j,c} / sqrt(head_dim),  LSE = ln sum_j exp(s_j),
+ *   O   = sum_j exp(s_j - LSE) v_{j,c}.
+ * O: device bf16 [n][num_q_heads][head_dim]; LSE: device fp32
+ * [n][num_q_heads], natural log. Q, O 16-byte aligned, LSE 4-byte aligned.
+ * Each path segment shared by several listed leaves is read from HBM once
+ * for all of them. n == 0 is a no-op. Asynchronous on the tree's stream.
+ * Errors: TP_ERR_BAD_NODE, TP_ERR_NOT_LEAF, TP_ERR_EMPTY_PATH,
+ * TP_ERR_INVALID_ARG, TP_ERR_OOM / TP_ERR_CUDA (library scratch).
+ */
+tp_status tp_decode(tp_tree* tree, const tp_node* leaves, int32_t n, const void* Q, void* O,
+                    float* LSE);
+
+/* tp_decode with options (bit flags below). */
+#define TP_DECODE_NO_SHARE 1u        /* schedule every leaf's whole path on its own  */
+#define TP_DECODE_SMALL_ON_TENSOR 2u /* groups of < 16 query rows on the tensor-core */
+                                     /* kernel too (default: CUDA-core kernel)       */
+#define TP_DECODE_NO_CACHE 4u        /* rebuild the schedule even if cached          */
+tp_status tp_decode_ex(tp_tree* tree, const tp_node* leaves, int32_t n, const void* Q, void* O,
+                       float* LSE, uint32_t flags);
+
+/* Wait for the tree's stream; TP_ERR_DEVICE if a kernel gave up a bounded
+ * wait since the last tp_sync (the flag is then cleared), TP_ERR_CUDA on a
+ * CUDA error. */
+tp_status tp_sync(tp_tree* tree);
+
+/* Message for the last failed call on `tree` (or of tp_tree_create when
+ * tree == NULL). Valid until the next call on that tree. */
+const char* tp_last_error(tp_tree* tree);
+
+/* Node state. state: 0 live leaf, 1 frozen interior, 2 dead. */
+typedef struct {
+    tp_node parent; /* -1 for a root */
+    int32_t state;
+    int32_t n_tokens;
+    int32_t n_live_children;
+    int64_t path_tokens; /* tokens on the root-to-node path */
+} tp_node_info;
+tp_status tp_get_node_info(tp_tree* tree, tp_node node, tp_node_info* out);
+
+/* Pool and forest counters. */
+typedef struct {
+    int64_t pool_blocks;
+    int64_t free_blocks;
+    int64_t live_nodes;
+    int64_t total_nodes;
+} tp_stats;
+tp_status tp_get_stats(tp_tree* tree, tp_stats* out);
+
+/* ---- kernel timing ------------------------------------------------------
+ * While profiling is on, every kernel the library launches is bracketed by a
+ * pair of CUDA events recorded on the tree's stream. tp_profile_stop waits
+ * for the stream and returns, per kernel kind, the launch count and the sum
+ * of the event-measured durations. Index: 0 decode attention, 1 LSE merge,
+ * 2 append copy, 3 inspection gather. */
+#define TP_KERNEL_KINDS 4
+typedef struct {
+    int64_t launches[TP_KERNEL_KINDS];
+    double milliseconds[TP_KERNEL_KINDS];
+} tp_kernel_times;
+tp_status tp_profile_start(tp_tree* tree);
+tp_status tp_profile_stop(tp_tree* tree, tp_kernel_times* out);
+
+/* ---- inspection (tests and tools) ------------------------------------ */
+
+/* Pool slot of every token on leaf's root-to-leaf path, root first.
+ * slots: host int64 [cap]; *n receives the path length (slots untouched
+ * beyond cap; TP_ERR_INVALID_ARG if cap < length). */
+tp_status tp_debug_path(tp_tree* tree, tp_node leaf, int64_t* slots, int64_t cap, int64_t* n);
+
+/* Copy leaf's path K and V out of the pool on the device, through the same
+ * block tables the decode kernels read. K_out, V_out: device bf16
+ * [cap_tokens][num_kv_heads][head_dim], 16-byte aligned; *n receives the
+ * path length (TP_ERR_INVALID_ARG if cap_tokens < length). */
+tp_status tp_debug_gather(tp_tree* tree, tp_node leaf, void* K_out, void* V_out,
+                          int64_t cap_tokens, int64_t* n);
+
+/*
+ * The decode schedule tp_decode_ex(flags) would run, as int32 words in host
+ * buf[cap]; *len receives the word count (TP_ERR_INVALID_ARG if cap is too
+ * small; call with cap 0 to size). Layout:
+ *   [0] magic 0x54505344, [1] n_units, [2] n_tiles, [3] n_occ_entries,
+ *   [4] n (leaf occurrences), [5] n_slots, [6] n_merge_entries, [7] group g,
+ *   [8] n_tensor_units, [9..15] reserved (0),
+ *   then units  [n_units][8]: tile_off, n_tiles, occ_off, row0, n_rows,
+ *                             slot_base, kv_head, kind (0 CUDA-core, 1 tensor),
+ *   then tiles  [n_tiles]: block << 7 | (valid_tokens - 1),
+ *   then occ    [n_occ_entries]: leaf occurrence index (row i of Q),
+ *   then merge_off [n + 1], then merge_slot [n_merge_entries].
+ * Unit row r (0 <= r < n_rows) is item row row0 + r = p * g + j: occurrence
+ * occ[occ_off + p], q-head kv_head * g + j, written to partial slot
+ * slot_base + p. Occurrence i merges slots merge_slot[merge_off[i] ..
+ * merge_off[i+1]).
+ */
+tp_status tp_debug_schedule(tp_tree* tree, const tp_node* leaves, int32_t n, uint32_t flags,
+                            int32_t* buf, int64_t cap, int64_t* len);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TREEPO_H_ */

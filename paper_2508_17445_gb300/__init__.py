@@ -1,0 +1,364 @@
+"""Python binding of libtreepo: decode attention over a segment tree of KV
+caches on one GB300 (sm_103a).
+
+Every function here has the name of the C entry point it calls (declared in
+``include/treepo.h``) and only marshals arguments: tensors become device
+pointers, node lists become int32 host arrays, status codes become
+``TreepoError``. All computation happens in the library's CUDA kernels; when
+the library is missing this module raises instead of falling back.
+
+``Forest`` is a small owner object: it allocates the pool arena with PyTorch
+(PyTorch is used for device memory and streams only) and frees the tree.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Dict, Iterable, List, Optional, Sequence
+
+import numpy as np
+
+__all__ = [
+    "TreepoError", "load_library", "library_path", "tp_pool_bytes", "tp_tree_create", "tp_tree_destroy",
+    "tp_set_stream", "tp_add_root", "tp_append_segment", "tp_fork", "tp_prune", "tp_decode", "tp_decode_ex",
+    "tp_sync", "tp_last_error", "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop",
+    "tp_debug_path", "tp_debug_gather",
+    "tp_debug_schedule", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_SMALL_ON_TENSOR", "TP_DECODE_NO_CACHE",
+    "EXPORTED_SYMBOLS",
+]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_HERE, "libtreepo.so")
+_lib: Optional[ctypes.CDLL] = None
+
+TP_DECODE_NO_SHARE = 1
+TP_DECODE_SMALL_ON_TENSOR = 2
+TP_DECODE_NO_CACHE = 4
+
+STATUS_NAMES = {0: "OK", -1: "INVALID_ARG", -2: "OOM", -3: "BAD_NODE", -4: "FROZEN", -5: "NOT_LEAF",
+                -6: "EMPTY_PATH", -7: "CUDA", -8: "DEVICE"}
+
+EXPORTED_SYMBOLS = (
+    "tp_pool_bytes", "tp_tree_create", "tp_tree_destroy", "tp_set_stream", "tp_add_root",
+    "tp_append_segment", "tp_fork", "tp_prune", "tp_decode", "tp_decode_ex", "tp_sync", "tp_last_error",
+    "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop", "tp_debug_path",
+    "tp_debug_gather", "tp_debug_schedule",
+)
+
+
+class TreepoError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        self.status = status
+        self.code = STATUS_NAMES.get(status, str(status))
+        super().__init__(f"TP_ERR_{self.code}: {message}")
+
+
+class TpConfig(ctypes.Structure):
+    _fields_ = [("num_q_heads", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("block_tokens", ctypes.c_int32),
+                ("pool_blocks", ctypes.c_int64), ("pool", ctypes.c_void_p), ("cuda_stream", ctypes.c_void_p)]
+
+
+class TpNodeInfo(ctypes.Structure):
+    _fields_ = [("parent", ctypes.c_int32), ("state", ctypes.c_int32), ("n_tokens", ctypes.c_int32),
+                ("n_live_children", ctypes.c_int32), ("path_tokens", ctypes.c_int64)]
+
+
+class TpKernelTimes(ctypes.Structure):
+    _fields_ = [("launches", ctypes.c_int64 * 4), ("milliseconds", ctypes.c_double * 4)]
+
+
+KERNEL_KINDS = ("decode", "merge", "append", "gather")
+
+
+class TpStats(ctypes.Structure):
+    _fields_ = [("pool_blocks", ctypes.c_int64), ("free_blocks", ctypes.c_int64),
+                ("live_nodes", ctypes.c_int64), ("total_nodes", ctypes.c_int64)]
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def load_library() -> ctypes.CDLL:
+    """Load libtreepo.so (built in-tree by ``paper_2508_17445_gb300.build``)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(_LIB_PATH):
+        raise ImportError(f"{_LIB_PATH} is missing: run `python -m paper_2508_17445_gb300.build` "
+                          "(there is no fallback implementation)")
+    lib = ctypes.CDLL(_LIB_PATH)
+    P, I32, I64, U32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32
+    sig = {
+        "tp_pool_bytes": (I64, [P]),
+        "tp_tree_create": (I32, [P, P]),
+        "tp_tree_destroy": (I32, [P]),
+        "tp_set_stream": (I32, [P, P]),
+        "tp_add_root": (I32, [P, P]),
+        "tp_append_segment": (I32, [P, I32, I32, P, P]),
+        "tp_fork": (I32, [P, I32, I32, P]),
+        "tp_prune": (I32, [P, I32]),
+        "tp_decode": (I32, [P, P, I32, P, P, P]),
+        "tp_decode_ex": (I32, [P, P, I32, P, P, P, U32]),
+        "tp_sync": (I32, [P]),
+        "tp_last_error": (ctypes.c_char_p, [P]),
+        "tp_get_node_info": (I32, [P, I32, P]),
+        "tp_get_stats": (I32, [P, P]),
+        "tp_profile_start": (I32, [P]),
+        "tp_profile_stop": (I32, [P, P]),
+        "tp_debug_path": (I32, [P, I32, P, I64, P]),
+        "tp_debug_gather": (I32, [P, I32, P, P, I64, P]),
+        "tp_debug_schedule": (I32, [P, P, I32, U32, P, I64, P]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _check(handle, status: int) -> None:
+    if status != 0:
+        msg = load_library().tp_last_error(handle)
+        raise TreepoError(status, msg.decode() if msg else "")
+
+
+def _ptr(t) -> Optional[int]:
+    if t is None:
+        return None
+    return t.data_ptr()
+
+
+def _node_array(nodes: Sequence[int]) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(nodes, dtype=np.int32).reshape(-1))
+
+
+# ---------------------------------------------------------------- C calls --
+def tp_pool_bytes(cfg: TpConfig) -> int:
+    return int(load_library().tp_pool_bytes(ctypes.byref(cfg)))
+
+
+def tp_tree_create(cfg: TpConfig) -> ctypes.c_void_p:
+    h = ctypes.c_void_p()
+    _check(None, load_library().tp_tree_create(ctypes.byref(cfg), ctypes.byref(h)))
+    return h
+
+
+def tp_tree_destroy(h) -> None:
+    _check(None, load_library().tp_tree_destroy(h))
+
+
+def tp_set_stream(h, stream_ptr: int) -> None:
+    _check(h, load_library().tp_set_stream(h, stream_ptr))
+
+
+def tp_add_root(h) -> int:
+    out = ctypes.c_int32()
+    _check(h, load_library().tp_add_root(h, ctypes.byref(out)))
+    return out.value
+
+
+def tp_append_segment(h, node: int, n_tokens: int, K=None, V=None) -> None:
+    """K, V: device bf16 [n_tokens][Hkv][hd] tensors (None on a metadata-only tree)."""
+    _check(h, load_library().tp_append_segment(h, node, n_tokens, _ptr(K), _ptr(V)))
+
+
+def tp_fork(h, node: int, k: int) -> List[int]:
+    out = (ctypes.c_int32 * max(k, 1))()
+    _check(h, load_library().tp_fork(h, node, k, out))
+    return list(out[:k])
+
+
+def tp_prune(h, leaf: int) -> None:
+    _check(h, load_library().tp_prune(h, leaf))
+
+
+def tp_decode_ex(h, leaves: Sequence[int], Q, O, LSE, flags: int = 0) -> None:
+    arr = _node_array(leaves)
+    _check(h, load_library().tp_decode_ex(h, arr.ctypes.data, len(arr), _ptr(Q), _ptr(O), _ptr(LSE), flags))
+
+
+def tp_decode(h, leaves: Sequence[int], Q, O, LSE) -> None:
+    arr = _node_array(leaves)
+    _check(h, load_library().tp_decode(h, arr.ctypes.data, len(arr), _ptr(Q), _ptr(O), _ptr(LSE)))
+
+
+def tp_sync(h) -> None:
+    _check(h, load_library().tp_sync(h))
+
+
+def tp_last_error(h) -> str:
+    m = load_library().tp_last_error(h)
+    return m.decode() if m else ""
+
+
+def tp_get_node_info(h, node: int) -> Dict[str, int]:
+    info = TpNodeInfo()
+    _check(h, load_library().tp_get_node_info(h, node, ctypes.byref(info)))
+    return {f: getattr(info, f) for f, _ in TpNodeInfo._fields_}
+
+
+def tp_get_stats(h) -> Dict[str, int]:
+    st = TpStats()
+    _check(h, load_library().tp_get_stats(h, ctypes.byref(st)))
+    return {f: getattr(st, f) for f, _ in TpStats._fields_}
+
+
+def tp_profile_start(h) -> None:
+    _check(h, load_library().tp_profile_start(h))
+
+
+def tp_profile_stop(h) -> Dict[str, Dict[str, float]]:
+    """{kernel kind: {"launches": n, "ms": summed event time}}."""
+    kt = TpKernelTimes()
+    _check(h, load_library().tp_profile_stop(h, ctypes.byref(kt)))
+    return {k: {"launches": int(kt.launches[i]), "ms": float(kt.milliseconds[i])} for i, k in enumerate(KERNEL_KINDS)}
+
+
+def tp_debug_path(h, leaf: int) -> np.ndarray:
+    n = ctypes.c_int64()
+    lib = load_library()
+    info = tp_get_node_info(h, leaf)
+    cap = max(int(info["path_tokens"]), 1)
+    out = np.zeros(cap, dtype=np.int64)
+    _check(h, lib.tp_debug_path(h, leaf, out.ctypes.data, cap, ctypes.byref(n)))
+    return out[: n.value]
+
+
+def tp_debug_gather(h, leaf: int, K_out, V_out) -> int:
+    n = ctypes.c_int64()
+    _check(h, load_library().tp_debug_gather(h, leaf, _ptr(K_out), _ptr(V_out), K_out.shape[0], ctypes.byref(n)))
+    return n.value
+
+
+def tp_debug_schedule(h, leaves: Sequence[int], flags: int = 0) -> Dict[str, np.ndarray]:
+    """The schedule tp_decode_ex(flags) would run, decoded into arrays."""
+    arr = _node_array(leaves)
+    lib = load_library()
+    n_words = ctypes.c_int64()
+    _check(h, lib.tp_debug_schedule(h, arr.ctypes.data if len(arr) else None, len(arr), flags, None, 0,
+                                     ctypes.byref(n_words)))
+    buf = np.zeros(max(n_words.value, 1), dtype=np.int32)
+    _check(h, lib.tp_debug_schedule(h, arr.ctypes.data if len(arr) else None, len(arr), flags,
+                                     buf.ctypes.data, len(buf), ctypes.byref(n_words)))
+    w = buf[: n_words.value]
+    assert w[0] == 0x54505344
+    n_units, n_tiles, n_occ, n, n_slots, n_merge, g, n_tensor = (int(x) for x in w[1:9])
+    off = 16
+    units = w[off: off + 8 * n_units].reshape(n_units, 8)
+    off += 8 * n_units
+    tiles = w[off: off + n_tiles]
+    off += n_tiles
+    occ = w[off: off + n_occ]
+    off += n_occ
+    merge_off = w[off: off + n + 1]
+    off += n + 1
+    merge_slot = w[off: off + n_merge]
+    return {"units": units, "tiles": tiles, "occ": occ, "merge_off": merge_off, "merge_slot": merge_slot,
+            "n_slots": n_slots, "group": g, "n_tensor_units": n_tensor, "words": w}
+
+
+# ------------------------------------------------------------------ owner --
+class Forest:
+    """A tp_tree plus the pool arena it owns.
+
+    ``device=None`` builds a metadata-only tree (no CUDA, no pool): the host
+    logic runs, appends copy nothing, decode is refused.
+    """
+
+    def __init__(self, num_q_heads: int, num_kv_heads: int, head_dim: int, pool_blocks: int,
+                 block_tokens: int = 32, device=None, stream=None):
+        self.cfg = TpConfig(num_q_heads, num_kv_heads, head_dim, block_tokens, pool_blocks, None, None)
+        self.device = device
+        self.pool = None
+        if device is not None:
+            import torch
+            nbytes = tp_pool_bytes(self.cfg)
+            if nbytes <= 0:
+                raise TreepoError(-1, "bad tree configuration")
+            self.pool = torch.empty(nbytes, dtype=torch.uint8, device=device)
+            self.cfg.pool = self.pool.data_ptr()
+            s = stream if stream is not None else torch.cuda.current_stream(device)
+            self.cfg.cuda_stream = s.cuda_stream
+        self.handle = tp_tree_create(self.cfg)
+
+    def close(self) -> None:
+        if getattr(self, "handle", None) is not None:
+            tp_tree_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    # thin methods
+    def add_root(self) -> int:
+        return tp_add_root(self.handle)
+
+    def append(self, node: int, K=None, V=None, n_tokens: Optional[int] = None) -> None:
+        n = int(K.shape[0]) if K is not None else int(n_tokens)
+        tp_append_segment(self.handle, node, n, K, V)
+
+    def fork(self, node: int, k: int) -> List[int]:
+        return tp_fork(self.handle, node, k)
+
+    def prune(self, leaf: int) -> None:
+        tp_prune(self.handle, leaf)
+
+    def decode(self, leaves: Sequence[int], Q, flags: int = 0, out=None):
+        import torch
+        n, hq, hd = Q.shape
+        if out is None:
+            O = torch.empty((n, hq, hd), dtype=torch.bfloat16, device=Q.device)
+            LSE = torch.empty((n, hq), dtype=torch.float32, device=Q.device)
+        else:
+            O, LSE = out
+        tp_decode_ex(self.handle, leaves, Q, O, LSE, flags)
+        return O, LSE
+
+    def sync(self) -> None:
+        tp_sync(self.handle)
+
+    def stats(self) -> Dict[str, int]:
+        return tp_get_stats(self.handle)
+
+    def node_info(self, node: int) -> Dict[str, int]:
+        return tp_get_node_info(self.handle, node)
+
+    def replay(self, ops: Iterable[tuple], kv_fn=None) -> Dict[int, int]:
+        """Apply a script of tree operations; returns script id -> node id.
+
+        ops: ("root", sid) | ("append", sid, kv_id, n) | ("fork", sid, (c..)) |
+        ("prune", sid). kv_fn(kv_id) -> (K, V) device tensors; with no kv_fn
+        (metadata-only tree) appends carry no data.
+        """
+        ids: Dict[int, int] = {}
+        for op in ops:
+            kind = op[0]
+            if kind == "root":
+                ids[op[1]] = self.add_root()
+            elif kind == "append":
+                if kv_fn is None:
+                    tp_append_segment(self.handle, ids[op[1]], op[3], None, None)
+                else:
+                    K, V = kv_fn(op[2])
+                    self.append(ids[op[1]], K, V)
+            elif kind == "fork":
+                kids = self.fork(ids[op[1]], len(op[2]))
+                for sid, nid in zip(op[2], kids):
+                    ids[sid] = nid
+            elif kind == "prune":
+                self.prune(ids[op[1]])
+            else:
+                raise ValueError(f"unknown op {kind!r}")
+        return ids

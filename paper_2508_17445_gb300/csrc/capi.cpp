@@ -1,0 +1,494 @@
+// capi.cpp -- the extern "C" entry points declared in include/treepo.h.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <new>
+#include <string>
+
+#include "forest.h"
+
+using tp::fail;
+
+namespace {
+
+thread_local std::string g_create_err;
+
+bool aligned(const void* p, uintptr_t a) { return ((uintptr_t)p % a) == 0; }
+
+tp_status cuda_fail(tp_tree* t, cudaError_t e, const char* what) {
+    return fail(t, TP_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+// Grow a device buffer; waits for the stream so no queued kernel still reads it.
+template <typename T>
+tp_status ensure_device(tp_tree* t, T*& ptr, int64_t& cap, int64_t need, const char* what) {
+    if (need <= cap) return TP_OK;
+    int64_t want = std::max<int64_t>(need, cap + cap / 2);
+    if (ptr) {
+        cudaStreamSynchronize(t->stream);
+        cudaFree(ptr);
+        ptr = nullptr;
+        cap = 0;
+    }
+    cudaError_t e = cudaMalloc((void**)&ptr, (size_t)want * sizeof(T));
+    if (e != cudaSuccess) {
+        ptr = nullptr;
+        cudaGetLastError();
+        return fail(t, e == cudaErrorMemoryAllocation ? TP_ERR_OOM : TP_ERR_CUDA,
+                    std::string(what) + ": " + cudaGetErrorString(e));
+    }
+    cap = want;
+    return TP_OK;
+}
+
+// Copy a schedule to the device through a double-buffered pinned staging area.
+tp_status upload_schedule(tp_tree* t, const tp::Schedule& s) {
+    const int64_t words = (int64_t)s.words.size();
+    tp_status st = ensure_device(t, t->d_sched, t->d_sched_cap, words, "schedule buffer");
+    if (st != TP_OK) return st;
+    const int k = t->pinned_next;
+    t->pinned_next ^= 1;
+    if (t->h_pinned_ev[k] == nullptr) {
+        cudaError_t e = cudaEventCreateWithFlags(&t->h_pinned_ev[k], cudaEventDisableTiming);
+        if (e != cudaSuccess) return cuda_fail(t, e, "cudaEventCreate");
+    }
+    cudaError_t e = cudaEventSynchronize(t->h_pinned_ev[k]);  // previous copy out of this buffer done
+    if (e != cudaSuccess) return cuda_fail(t, e, "cudaEventSynchronize");
+    if (t->h_pinned_cap[k] < words) {
+        if (t->h_pinned[k]) cudaFreeHost(t->h_pinned[k]);
+        t->h_pinned[k] = nullptr;
+        t->h_pinned_cap[k] = 0;
+        int64_t want = std::max<int64_t>(words, 1 << 16);
+        e = cudaHostAlloc((void**)&t->h_pinned[k], (size_t)want * 4, cudaHostAllocDefault);
+        if (e != cudaSuccess) return cuda_fail(t, e, "cudaHostAlloc");
+        t->h_pinned_cap[k] = want;
+    }
+    std::memcpy(t->h_pinned[k], s.words.data(), (size_t)words * 4);
+    e = cudaMemcpyAsync(t->d_sched, t->h_pinned[k], (size_t)words * 4, cudaMemcpyHostToDevice, t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "schedule upload");
+    e = cudaEventRecord(t->h_pinned_ev[k], t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "cudaEventRecord");
+    return TP_OK;
+}
+
+cudaEvent_t next_event(tp_tree* t) {
+    if (t->ev_used == t->ev_pool.size()) {
+        cudaEvent_t e = nullptr;
+        if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+        t->ev_pool.push_back(e);
+    }
+    return t->ev_pool[t->ev_used++];
+}
+
+}  // namespace
+
+namespace tp {
+LaunchTimer::LaunchTimer(tp_tree* t, int kind) : t_(t), kind_(kind) {
+    if (!t_->profiling) return;
+    cudaEvent_t a = next_event(t_);
+    b_ = next_event(t_);
+    if (!a || !b_) {
+        b_ = nullptr;
+        return;
+    }
+    cudaEventRecord(a, t_->stream);
+    t_->timed.push_back({kind_, a, b_});
+}
+LaunchTimer::~LaunchTimer() {
+    if (b_) cudaEventRecord(b_, t_->stream);
+}
+}  // namespace tp
+
+extern "C" {
+
+int64_t tp_pool_bytes(const tp_config* c) {
+    if (!c || c->num_kv_heads < 1 || c->head_dim < 1 || c->block_tokens < 1 || c->pool_blocks < 1) return -1;
+    return c->pool_blocks * 2 * (int64_t)c->num_kv_heads * c->block_tokens * c->head_dim * 2;
+}
+
+tp_status tp_tree_create(const tp_config* cfg, tp_tree** out) {
+    if (!out) return TP_ERR_INVALID_ARG;
+    *out = nullptr;
+    auto bad = [](const char* m) {
+        g_create_err = m;
+        return TP_ERR_INVALID_ARG;
+    };
+    if (!cfg) return bad("cfg is NULL");
+    if (cfg->num_q_heads < 1 || cfg->num_kv_heads < 1 || cfg->num_q_heads % cfg->num_kv_heads)
+        return bad("num_q_heads must be a positive multiple of num_kv_heads");
+    if (cfg->head_dim != 64 && cfg->head_dim != 128) return bad("head_dim must be 64 or 128");
+    if (cfg->block_tokens != 32) return bad("block_tokens must be 32");
+    if (cfg->pool_blocks < 1 || cfg->pool_blocks > tp::kMaxPoolBlocks) return bad("pool_blocks must be in [1, 2^24]");
+    if (cfg->pool && !aligned(cfg->pool, 256)) return bad("pool must be 256-byte aligned");
+    tp_tree* t = new (std::nothrow) tp_tree();
+    if (!t) {
+        g_create_err = "out of host memory";
+        return TP_ERR_OOM;
+    }
+    t->cfg = *cfg;
+    t->stream = (cudaStream_t)cfg->cuda_stream;
+    t->pool.init(cfg->pool_blocks);
+    if (cfg->pool) {
+        cudaError_t e = cudaMalloc((void**)&t->d_err, sizeof(int32_t));
+        if (e == cudaSuccess) e = cudaMemsetAsync(t->d_err, 0, sizeof(int32_t), t->stream);
+        if (e != cudaSuccess) {
+            g_create_err = std::string("device error flag: ") + cudaGetErrorString(e);
+            cudaGetLastError();
+            if (t->d_err) cudaFree(t->d_err);
+            delete t;
+            return TP_ERR_CUDA;
+        }
+    }
+    *out = t;
+    return TP_OK;
+}
+
+tp_status tp_tree_destroy(tp_tree* t) {
+    if (!t) return TP_OK;
+    if (t->cfg.pool) cudaStreamSynchronize(t->stream);
+    if (t->d_err) cudaFree(t->d_err);
+    if (t->d_sched) cudaFree(t->d_sched);
+    if (t->d_part) cudaFree(t->d_part);
+    if (t->d_gather_tiles) cudaFree(t->d_gather_tiles);
+    for (cudaEvent_t e : t->ev_pool) cudaEventDestroy(e);
+    for (int k = 0; k < 2; ++k) {
+        if (t->h_pinned[k]) cudaFreeHost(t->h_pinned[k]);
+        if (t->h_pinned_ev[k]) cudaEventDestroy(t->h_pinned_ev[k]);
+    }
+    delete t;
+    return TP_OK;
+}
+
+tp_status tp_set_stream(tp_tree* t, void* stream) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    t->stream = (cudaStream_t)stream;
+    return TP_OK;
+}
+
+tp_status tp_add_root(tp_tree* t, tp_node* out) {
+    if (!t || !out) return TP_ERR_INVALID_ARG;
+    if (t->nodes.size() >= (size_t)INT32_MAX) return fail(t, TP_ERR_OOM, "node ids exhausted");
+    t->nodes.emplace_back();
+    *out = (tp_node)t->nodes.size() - 1;
+    ++t->live_nodes;
+    ++t->version;
+    return TP_OK;
+}
+
+tp_status tp_append_segment(tp_tree* t, tp_node node, int32_t n_tokens, const void* K, const void* V) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    tp_status st = tp::check_live(t, node, false);
+    if (st != TP_OK) return st;
+    tp::Node& nd = t->nodes[(size_t)node];
+    if (nd.state != 0) return fail(t, TP_ERR_FROZEN, "node " + std::to_string(node) + " has been forked");
+    if (n_tokens < 0) return fail(t, TP_ERR_INVALID_ARG, "n_tokens < 0");
+    if (n_tokens == 0) return TP_OK;
+    if ((int64_t)nd.n_tokens + n_tokens > INT32_MAX / 2) return fail(t, TP_ERR_INVALID_ARG, "node too long");
+    if (t->cfg.pool) {
+        if (!K || !V || !aligned(K, 16) || !aligned(V, 16))
+            return fail(t, TP_ERR_INVALID_ARG, "K and V must be non-NULL 16-byte aligned device pointers");
+    } else if (K || V) {
+        return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree: K and V must be NULL");
+    }
+    const int32_t bt = t->cfg.block_tokens;
+    const int64_t need = ((int64_t)nd.n_tokens + n_tokens + bt - 1) / bt - (int64_t)nd.blocks.size();
+    const size_t old_blocks = nd.blocks.size();
+    if (need > 0 && !t->pool.alloc(need, nd.blocks))
+        return fail(t, TP_ERR_OOM, "pool exhausted: need " + std::to_string(need) + " blocks, " +
+                                       std::to_string(t->pool.free_count()) + " free");
+    if (t->cfg.pool) {
+        const int32_t hkv = t->cfg.num_kv_heads, hd = t->cfg.head_dim;
+        tp::AppendArgs a;
+        a.pool = (uint8_t*)t->cfg.pool;
+        a.head_bytes = bt * hd * 2;
+        a.block_bytes = (int64_t)2 * hkv * a.head_bytes;
+        a.hkv = hkv;
+        const int64_t row_bytes = (int64_t)hkv * hd * 2;
+        int64_t pos = nd.n_tokens;
+        const int64_t end = (int64_t)nd.n_tokens + n_tokens;
+        while (pos < end) {
+            const int64_t bi = pos / bt;
+            const int64_t stop = std::min<int64_t>(end, (bi + tp::kAppendMaxBlocks) * bt);
+            a.first_row = (int32_t)(pos % bt);
+            a.n_tokens = (int32_t)(stop - pos);
+            const int64_t nb = (stop - 1) / bt - bi + 1;
+            for (int64_t b = 0; b < nb; ++b) a.blocks[b] = nd.blocks[(size_t)(bi + b)];
+            a.k = (const uint8_t*)K + (pos - nd.n_tokens) * row_bytes;
+            a.v = (const uint8_t*)V + (pos - nd.n_tokens) * row_bytes;
+            cudaError_t e;
+            {
+                tp::LaunchTimer timer(t, tp::KK_APPEND);
+                e = tp::launch_append(hd, a, t->stream);
+            }
+            if (e != cudaSuccess) {
+                std::vector<int32_t> fresh(nd.blocks.begin() + (long)old_blocks, nd.blocks.end());
+                nd.blocks.resize(old_blocks);
+                t->pool.release(fresh);
+                return cuda_fail(t, e, "append kernel");
+            }
+            pos = stop;
+        }
+    }
+    nd.n_tokens += n_tokens;
+    ++t->version;
+    return TP_OK;
+}
+
+tp_status tp_fork(tp_tree* t, tp_node node, int32_t k, tp_node* out_children) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    tp_status st = tp::check_live(t, node, false);
+    if (st != TP_OK) return st;
+    if (k < 1) return fail(t, TP_ERR_INVALID_ARG, "fork needs k >= 1");
+    if (!out_children) return fail(t, TP_ERR_INVALID_ARG, "out_children is NULL");
+    if (t->nodes.size() + (size_t)k > (size_t)INT32_MAX) return fail(t, TP_ERR_OOM, "node ids exhausted");
+    const int64_t before = t->nodes[(size_t)node].path_before + t->nodes[(size_t)node].n_tokens;
+    for (int32_t c = 0; c < k; ++c) {
+        tp::Node child;
+        child.parent = node;
+        child.path_before = before;
+        t->nodes.push_back(std::move(child));
+        out_children[c] = (tp_node)t->nodes.size() - 1;
+    }
+    tp::Node& nd = t->nodes[(size_t)node];
+    nd.state = 1;
+    nd.kids_live += k;
+    t->live_nodes += k;
+    ++t->version;
+    return TP_OK;
+}
+
+tp_status tp_prune(tp_tree* t, tp_node leaf) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    tp_status st = tp::check_live(t, leaf, true);
+    if (st != TP_OK) return st;
+    int32_t x = leaf;
+    while (true) {
+        tp::Node& nd = t->nodes[(size_t)x];
+        t->pool.release(nd.blocks);
+        nd.blocks.clear();
+        nd.blocks.shrink_to_fit();
+        nd.state = 2;
+        --t->live_nodes;
+        x = nd.parent;
+        if (x == -1) break;
+        if (--t->nodes[(size_t)x].kids_live > 0) break;
+    }
+    ++t->version;
+    return TP_OK;
+}
+
+tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void* Q, void* O, float* LSE,
+                       uint32_t flags) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    if (n < 0) return fail(t, TP_ERR_INVALID_ARG, "n < 0");
+    if (n == 0) return TP_OK;
+    if (!leaves) return fail(t, TP_ERR_INVALID_ARG, "leaves is NULL");
+    if (!t->cfg.pool) return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree cannot decode");
+    if (!Q || !O || !LSE || !aligned(Q, 16) || !aligned(O, 16) || !aligned(LSE, 4))
+        return fail(t, TP_ERR_INVALID_ARG, "Q/O must be 16-byte and LSE 4-byte aligned device pointers");
+    const uint32_t key_flags = flags & ~TP_DECODE_NO_CACHE;
+    const bool hit = !(flags & TP_DECODE_NO_CACHE) && t->sched_valid && t->sched_version == t->version &&
+                     t->sched_flags == key_flags && t->sched_leaves.size() == (size_t)n &&
+                     std::equal(leaves, leaves + n, t->sched_leaves.begin());
+    tp::Schedule& S = t->sched;
+    if (!hit) {
+        t->sched_valid = false;
+        tp_status st = tp::build_schedule(t, leaves, n, flags, S);
+        if (st != TP_OK) return st;
+        st = upload_schedule(t, S);
+        if (st != TP_OK) return st;
+        t->sched_valid = true;
+        t->sched_version = t->version;
+        t->sched_flags = key_flags;
+        t->sched_leaves.assign(leaves, leaves + n);
+    }
+    const int32_t hq = t->cfg.num_q_heads, hd = t->cfg.head_dim;
+    const int64_t part_floats = (int64_t)S.n_slots * hq * (hd + 1);
+    tp_status st = ensure_device(t, t->d_part, t->d_part_cap, std::max<int64_t>(part_floats, 1), "partial buffer");
+    if (st != TP_OK) return st;
+
+    tp::DecodeArgs a;
+    a.units = t->d_sched + S.off_units;
+    a.tiles = t->d_sched + S.off_tiles;
+    a.occ = t->d_sched + S.off_occ;
+    a.q = (const uint16_t*)Q;
+    a.pool = (const uint8_t*)t->cfg.pool;
+    a.part_o = t->d_part;
+    a.part_lse = t->d_part + (int64_t)S.n_slots * hq * hd;
+    a.err = t->d_err;
+    a.head_bytes = t->cfg.block_tokens * hd * 2;
+    a.block_bytes = (int64_t)2 * t->cfg.num_kv_heads * a.head_bytes;
+    a.n_units = S.n_units;
+    a.hq = hq;
+    a.hkv = t->cfg.num_kv_heads;
+    a.group = hq / t->cfg.num_kv_heads;
+    a.qk_scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
+    cudaError_t e = cudaSuccess;
+    if (a.n_units > 0) {
+        tp::LaunchTimer timer(t, tp::KK_DECODE);
+        e = tp::launch_decode(hd, a, t->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(t, e, "decode kernel");
+
+    tp::MergeArgs m;
+    m.merge_off = t->d_sched + S.off_merge_off;
+    m.merge_slot = t->d_sched + S.off_merge_slot;
+    m.part_o = a.part_o;
+    m.part_lse = a.part_lse;
+    m.out = (uint16_t*)O;
+    m.lse = LSE;
+    m.n = n;
+    m.hq = hq;
+    {
+        tp::LaunchTimer timer(t, tp::KK_MERGE);
+        e = tp::launch_merge(hd, m, t->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(t, e, "merge kernel");
+    return TP_OK;
+}
+
+tp_status tp_decode(tp_tree* t, const tp_node* leaves, int32_t n, const void* Q, void* O, float* LSE) {
+    return tp_decode_ex(t, leaves, n, Q, O, LSE, 0u);
+}
+
+tp_status tp_profile_start(tp_tree* t) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    if (!t->cfg.pool) return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree launches no kernels");
+    cudaError_t e = cudaStreamSynchronize(t->stream);  // recycled events must be idle
+    if (e != cudaSuccess) return cuda_fail(t, e, "cudaStreamSynchronize");
+    t->timed.clear();
+    t->ev_used = 0;
+    t->profiling = true;
+    return TP_OK;
+}
+
+tp_status tp_profile_stop(tp_tree* t, tp_kernel_times* out) {
+    if (!t || !out) return TP_ERR_INVALID_ARG;
+    t->profiling = false;
+    std::memset(out, 0, sizeof *out);
+    if (!t->cfg.pool) return TP_OK;
+    cudaError_t e = cudaStreamSynchronize(t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "cudaStreamSynchronize");
+    for (const auto& x : t->timed) {
+        float ms = 0.f;
+        e = cudaEventElapsedTime(&ms, x.a, x.b);
+        if (e != cudaSuccess) return cuda_fail(t, e, "cudaEventElapsedTime");
+        out->launches[x.kind] += 1;
+        out->milliseconds[x.kind] += ms;
+    }
+    t->timed.clear();
+    t->ev_used = 0;
+    return TP_OK;
+}
+
+tp_status tp_sync(tp_tree* t) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    if (!t->cfg.pool) return TP_OK;
+    cudaError_t e = cudaStreamSynchronize(t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "cudaStreamSynchronize");
+    int32_t flag = 0;
+    e = cudaMemcpy(&flag, t->d_err, sizeof flag, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(t, e, "error flag read");
+    if (flag) {
+        cudaMemset(t->d_err, 0, sizeof(int32_t));
+        return fail(t, TP_ERR_DEVICE, "a kernel gave up a bounded wait (flag " + std::to_string(flag) + ")");
+    }
+    return TP_OK;
+}
+
+const char* tp_last_error(tp_tree* t) { return t ? t->err.c_str() : g_create_err.c_str(); }
+
+tp_status tp_get_node_info(tp_tree* t, tp_node node, tp_node_info* out) {
+    if (!t || !out) return TP_ERR_INVALID_ARG;
+    if (node < 0 || node >= (tp_node)t->nodes.size()) return fail(t, TP_ERR_BAD_NODE, "unknown node id");
+    const tp::Node& nd = t->nodes[(size_t)node];
+    out->parent = nd.parent;
+    out->state = nd.state;
+    out->n_tokens = nd.n_tokens;
+    out->n_live_children = nd.kids_live;
+    out->path_tokens = nd.path_before + nd.n_tokens;
+    return TP_OK;
+}
+
+tp_status tp_get_stats(tp_tree* t, tp_stats* out) {
+    if (!t || !out) return TP_ERR_INVALID_ARG;
+    out->pool_blocks = t->pool.size();
+    out->free_blocks = t->pool.free_count();
+    out->live_nodes = t->live_nodes;
+    out->total_nodes = (int64_t)t->nodes.size();
+    return TP_OK;
+}
+
+tp_status tp_debug_path(tp_tree* t, tp_node leaf, int64_t* slots, int64_t cap, int64_t* n) {
+    if (!t || !n) return TP_ERR_INVALID_ARG;
+    tp_status st = tp::check_live(t, leaf, true);
+    if (st != TP_OK) return st;
+    const tp::Node& nd = t->nodes[(size_t)leaf];
+    const int64_t len = nd.path_before + nd.n_tokens;
+    *n = len;
+    if (cap < len || (len && !slots)) return fail(t, TP_ERR_INVALID_ARG, "slots buffer too small");
+    std::vector<int32_t> tiles;
+    tp::path_tiles(t, leaf, tiles);
+    const int32_t bt = t->cfg.block_tokens;
+    int64_t k = 0;
+    for (int32_t w : tiles) {
+        const int64_t blk = w >> tp::kTileValidBits;
+        const int32_t valid = (w & ((1 << tp::kTileValidBits) - 1)) + 1;
+        for (int32_t r = 0; r < valid; ++r) slots[k++] = blk * bt + r;
+    }
+    return TP_OK;
+}
+
+tp_status tp_debug_gather(tp_tree* t, tp_node leaf, void* K_out, void* V_out, int64_t cap_tokens, int64_t* n) {
+    if (!t || !n) return TP_ERR_INVALID_ARG;
+    tp_status st = tp::check_live(t, leaf, true);
+    if (st != TP_OK) return st;
+    if (!t->cfg.pool) return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree has no device pool");
+    const tp::Node& nd = t->nodes[(size_t)leaf];
+    const int64_t len = nd.path_before + nd.n_tokens;
+    *n = len;
+    if (cap_tokens < len) return fail(t, TP_ERR_INVALID_ARG, "output buffers too small");
+    if (len == 0) return TP_OK;
+    if (!K_out || !V_out || !aligned(K_out, 16) || !aligned(V_out, 16))
+        return fail(t, TP_ERR_INVALID_ARG, "K_out/V_out must be 16-byte aligned device pointers");
+    std::vector<int32_t> tiles;
+    tp::path_tiles(t, leaf, tiles);
+    st = ensure_device(t, t->d_gather_tiles, t->d_gather_cap, (int64_t)tiles.size(), "gather tiles");
+    if (st != TP_OK) return st;
+    cudaError_t e = cudaMemcpyAsync(t->d_gather_tiles, tiles.data(), tiles.size() * 4, cudaMemcpyHostToDevice, t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "gather tile upload");
+    tp::GatherArgs a;
+    a.tiles = t->d_gather_tiles;
+    a.pool = (const uint8_t*)t->cfg.pool;
+    a.k_out = K_out;
+    a.v_out = V_out;
+    a.head_bytes = t->cfg.block_tokens * t->cfg.head_dim * 2;
+    a.block_bytes = (int64_t)2 * t->cfg.num_kv_heads * a.head_bytes;
+    a.hkv = t->cfg.num_kv_heads;
+    a.n_tiles = (int32_t)tiles.size();
+    a.block_tokens = t->cfg.block_tokens;
+    {
+        tp::LaunchTimer timer(t, tp::KK_GATHER);
+        e = tp::launch_gather(t->cfg.head_dim, a, len, t->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(t, e, "gather kernel");
+    e = cudaStreamSynchronize(t->stream);  // the host tile list must outlive the copy
+    if (e != cudaSuccess) return cuda_fail(t, e, "gather sync");
+    return TP_OK;
+}
+
+tp_status tp_debug_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t flags, int32_t* buf, int64_t cap,
+                            int64_t* len) {
+    if (!t || !len) return TP_ERR_INVALID_ARG;
+    if (n < 0 || (n > 0 && !leaves)) return fail(t, TP_ERR_INVALID_ARG, "bad leaf list");
+    tp::Schedule S;
+    tp_status st = tp::build_schedule(t, leaves, n, flags, S);
+    if (st != TP_OK) return st;
+    *len = (int64_t)S.words.size();
+    if (cap < *len) return cap == 0 ? TP_OK : fail(t, TP_ERR_INVALID_ARG, "buffer too small");
+    if (!buf) return fail(t, TP_ERR_INVALID_ARG, "buf is NULL");
+    std::memcpy(buf, S.words.data(), S.words.size() * 4);
+    return TP_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,830 @@
+// kernels.cu -- sm_103a kernels of libtreepo.
+//
+//   append_kernel   copy a segment's K/V into pool blocks (16-byte chunks,
+//                   XOR-swizzled inside each token row, see below)
+//   decode_kernel   split-KV flash-decode: one CTA per unit = (chunk of path
+//                   blocks, kv head, <= 64 stacked query rows). K/V blocks
+//                   stream through a shared-memory ring filled by TMA bulk
+//                   copies (cp.async.bulk + mbarrier transaction counts).
+//                   Units with < 16 rows (one leaf's GQA group, or two) run
+//                   on CUDA cores with warp-shuffle reductions; units whose
+//                   stacked rows form a real contraction run Q.K^T and P.V on
+//                   tensor cores (mma.sync m16n8k16 bf16 -> fp32).
+//   merge_kernel    per (leaf occurrence, q-head): log-sum-exp merge of the
+//                   partials of every unit on the path -> O (bf16), LSE (fp32)
+//   gather_kernel   inspection: copy a path's K/V out through the block tables
+//
+// Attention per row (q-head h of one leaf): s_j = q.k_j / sqrt(d),
+// LSE = ln sum_j exp(s_j), O = sum_j exp(s_j - LSE) v_j -- standard decode
+// attention over the root-to-leaf path, the trajectory s_1 (+) ... (+) s_j of
+// TreePO (Sec. 2.3). Scores are kept in the log2 domain (q.k * log2(e)/sqrt(d))
+// so exponentials are exp2; partial LSEs are log2, the final LSE is natural.
+//
+// Pool layout. Block b holds [K|V][kv head][32 tokens][d] bf16. Inside a
+// token row the 16-byte chunk c is stored at chunk position c ^ (row & 7), so
+// that ldmatrix row gathers (8 rows, same chunk) and the CUDA-core row reads
+// (one row, 8 chunks per quarter warp) both hit 8 distinct bank groups.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <algorithm>
+
+#include "forest.h"
+
+namespace tp {
+namespace {
+
+constexpr int kThreads = 128;      // 4 warps per CTA
+constexpr int kBlockTokens = 32;   // tokens per pool block (= tile)
+constexpr int kStageTokens = 64;   // two tiles per pipeline stage
+constexpr int kStages = 3;         // stages in the shared-memory ring
+constexpr uint64_t kWaitLimitNs = 2000000000ull;  // bounded mbarrier waits: 2 s
+
+// ------------------------------------------------------------ PTX helpers --
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+__device__ __forceinline__ float fast_exp2(float x) {  // ex2.approx: exp2(-inf) = +0
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Wait for an mbarrier phase with a time limit; false if the limit ran out.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 63) == 0 && global_ns() - t0 > kWaitLimitNs) return false;
+    }
+}
+
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+
+__device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// bf16 pair in a 32-bit word -> two fp32 (exact: bf16 is the top half of fp32)
+__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+__device__ __forceinline__ int swz(int row, int chunk) { return chunk ^ (row & 7); }
+
+// ------------------------------------------------------------------ append --
+template <int HD>
+__global__ void append_kernel(const AppendArgs a) {
+    constexpr int CH = HD / 8;  // 16-byte chunks per token row
+    const int64_t per_kv = (int64_t)a.n_tokens * a.hkv * CH;
+    const int64_t total = 2 * per_kv;
+    for (int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; idx < total;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        const int kv = idx >= per_kv;
+        const int64_t r = kv ? idx - per_kv : idx;
+        const int c = (int)(r % CH);
+        const int h = (int)((r / CH) % a.hkv);
+        const int i = (int)(r / ((int64_t)CH * a.hkv));
+        const uint4 val = reinterpret_cast<const uint4*>(kv ? a.v : a.k)[r];
+        const int pos = a.first_row + i;
+        const int blk = a.blocks[pos / kBlockTokens];
+        const int row = pos % kBlockTokens;
+        uint8_t* dst = a.pool + (int64_t)blk * a.block_bytes + (int64_t)(kv * a.hkv + h) * a.head_bytes +
+                       row * (HD * 2) + swz(row, c) * 16;
+        *reinterpret_cast<uint4*>(dst) = val;
+    }
+}
+
+// ------------------------------------------------------------------ gather --
+template <int HD>
+__global__ void gather_kernel(const GatherArgs a, int64_t n_tokens) {
+    constexpr int CH = HD / 8;
+    const int64_t per_kv = n_tokens * a.hkv * CH;
+    for (int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; idx < 2 * per_kv;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        const int kv = idx >= per_kv;
+        const int64_t r = kv ? idx - per_kv : idx;
+        const int c = (int)(r % CH);
+        const int h = (int)((r / CH) % a.hkv);
+        const int64_t tok = r / ((int64_t)CH * a.hkv);
+        // walk the tile list: tiles are full blocks except possibly the last
+        // block of each node, so locate the token by a linear scan
+        int64_t base = 0;
+        int32_t w = 0;
+        for (int k = 0; k < a.n_tiles; ++k) {
+            w = a.tiles[k];
+            const int valid = (w & ((1 << kTileValidBits) - 1)) + 1;
+            if (tok < base + valid) break;
+            base += valid;
+        }
+        const int row = (int)(tok - base);
+        const int64_t blk = w >> kTileValidBits;
+        const uint8_t* src = a.pool + blk * a.block_bytes + (int64_t)(kv * a.hkv + h) * a.head_bytes +
+                             row * (HD * 2) + swz(row, c) * 16;
+        reinterpret_cast<uint4*>(kv ? a.v_out : a.k_out)[r] = *reinterpret_cast<const uint4*>(src);
+    }
+}
+
+// ------------------------------------------------------------------ decode --
+struct UnitDesc {
+    int tile_off, n_tiles, occ_off, row0, n_rows, slot_base, kvh, kind;
+};
+
+template <int HD>
+struct Smem {
+    static constexpr int kRowBytes = HD * 2;
+    static constexpr int kHalfBytes = kStageTokens * kRowBytes;  // K or V of one stage
+    static constexpr int kStageBytes = 2 * kHalfBytes;
+    static constexpr int kBytes = kStages * kStageBytes;
+};
+
+// Shared pipeline bookkeeping of one CTA.
+struct Pipe {
+    uint64_t bars[kStages];  // "stage full" barriers (transaction counted)
+    int issued;              // tile pairs issued so far (written by thread 0)
+    int abort_at;            // first pair whose wait ran out, or -1
+};
+
+// Producer: issue the bulk copies of tile pair `pair` into stage `st`.
+template <int HD>
+__device__ __forceinline__ void issue_pair(const DecodeArgs& a, const UnitDesc& u, uint8_t* ring, uint32_t bar,
+                                           int pair, int st) {
+    constexpr int RB = HD * 2;
+    uint8_t* sk = ring + st * Smem<HD>::kStageBytes;
+    uint8_t* sv = sk + Smem<HD>::kHalfBytes;
+    uint32_t bytes = 0;
+    int32_t w[2];
+    int nt = 0;
+    for (int j = 0; j < 2; ++j) {
+        const int t = 2 * pair + j;
+        if (t < u.n_tiles) {
+            w[j] = a.tiles[u.tile_off + t];
+            bytes += 2u * (uint32_t)(((w[j] & ((1 << kTileValidBits) - 1)) + 1) * RB);
+            nt = j + 1;
+        }
+    }
+    mbar_arrive_expect_tx(bar, bytes);
+    for (int j = 0; j < nt; ++j) {
+        const int valid = (w[j] & ((1 << kTileValidBits) - 1)) + 1;
+        const int64_t blk = w[j] >> kTileValidBits;
+        const uint8_t* src = a.pool + blk * a.block_bytes + (int64_t)u.kvh * a.head_bytes;
+        bulk_g2s(smem_u32(sk + j * kBlockTokens * RB), src, valid * RB, bar);
+        bulk_g2s(smem_u32(sv + j * kBlockTokens * RB), src + (int64_t)a.hkv * a.head_bytes, valid * RB, bar);
+    }
+}
+
+__device__ __forceinline__ int tile_valid(const DecodeArgs& a, const UnitDesc& u, int t) {
+    return t < u.n_tiles ? (a.tiles[u.tile_off + t] & ((1 << kTileValidBits) - 1)) + 1 : 0;
+}
+
+// ---- CUDA-core path: <= 16 rows, 8 rows per warp ------------------------
+// Lane layout: LPT = HD/8 lanes share one token (8 dims each, one 16-byte
+// chunk), TPS = 32/LPT tokens per warp step. Dot products over the LPT lanes
+// of a token are finished by a transposing butterfly: each level halves the
+// number of rows a lane carries, so 8 rows cost 7 shuffles instead of 8x4.
+template <int HD>
+struct CudaCorePath {
+    static constexpr int LPT = HD / 8;
+    static constexpr int TPS = 32 / LPT;
+    static constexpr int NR = 8;
+
+    // acc[0..7] -> lane keeps one row's full sum; returns it.
+    __device__ __forceinline__ static float transpose_reduce(float (&acc)[NR], int lane) {
+        if (LPT == 16) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const bool up = lane & 8;
+                const float send = up ? acc[i] : acc[i + 4];
+                const float keep = up ? acc[i + 4] : acc[i];
+                acc[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+            }
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                const bool up = lane & 4;
+                const float send = up ? acc[i] : acc[i + 2];
+                const float keep = up ? acc[i + 2] : acc[i];
+                acc[i] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+            }
+            {
+                const bool up = lane & 2;
+                const float send = up ? acc[0] : acc[1];
+                const float keep = up ? acc[1] : acc[0];
+                acc[0] = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+            }
+            return acc[0] + __shfl_xor_sync(0xffffffffu, acc[0], 1);  // row (lane >> 1) & 7
+        } else {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const bool up = lane & 4;
+                const float send = up ? acc[i] : acc[i + 4];
+                const float keep = up ? acc[i + 4] : acc[i];
+                acc[i] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+            }
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                const bool up = lane & 2;
+                const float send = up ? acc[i] : acc[i + 2];
+                const float keep = up ? acc[i + 2] : acc[i];
+                acc[i] = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+            }
+            const bool up = lane & 1;
+            const float send = up ? acc[0] : acc[1];
+            const float keep = up ? acc[1] : acc[0];
+            return keep + __shfl_xor_sync(0xffffffffu, send, 1);  // row lane & 7
+        }
+    }
+    __device__ __forceinline__ static int reduce_row(int lane) { return LPT == 16 ? (lane >> 1) & 7 : lane & 7; }
+    __device__ __forceinline__ static bool reduce_writer(int lane) { return LPT == 16 ? (lane & 1) == 0 : true; }
+
+    __device__ static void run(const DecodeArgs& a, const UnitDesc& u, uint8_t* ring, Pipe* pp, float* scratch) {
+        volatile Pipe* vp = pp;
+        const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+        const int n_rg = (u.n_rows + NR - 1) / NR;  // 1 or 2 row groups
+        const int n_sp = 4 / n_rg;                  // token splits
+        const int rg = warp % n_rg, sp = warp / n_rg;
+        const int TW = kStageTokens / n_sp;  // tokens of a stage this warp handles
+        const int dg = lane % LPT, ts = lane / LPT;
+
+        // q rows of this warp, 8 dims per lane, pre-scaled to the log2 domain
+        float qf[NR][8];
+#pragma unroll
+        for (int r = 0; r < NR; ++r) {
+            const int rr = rg * NR + r;
+            if (rr < u.n_rows) {
+                const int item_row = u.row0 + rr;
+                const int occ = a.occ[u.occ_off + item_row / a.group];
+                const int qh = u.kvh * a.group + item_row % a.group;
+                const uint4 w = *reinterpret_cast<const uint4*>(a.q + ((int64_t)occ * a.hq + qh) * HD + dg * 8);
+                const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    qf[r][2 * k] = bf_lo(ww[k]) * a.qk_scale_log2;
+                    qf[r][2 * k + 1] = bf_hi(ww[k]) * a.qk_scale_log2;
+                }
+            } else {
+#pragma unroll
+                for (int k = 0; k < 8; ++k) qf[r][k] = 0.f;
+            }
+        }
+        float o[NR][8];
+#pragma unroll
+        for (int r = 0; r < NR; ++r)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) o[r][k] = 0.f;
+        // running max / sum of row (lane >> 2), replicated over its quad
+        float m_run = -INFINITY, l_run = 0.f;
+        float* sc = scratch + warp * (kStageTokens * NR);  // [token][row]
+
+        const int n_pairs = (u.n_tiles + 1) / 2;
+        for (int pr = 0; pr < n_pairs; ++pr) {
+            const int st = pr % kStages;
+            if (!mbar_wait(smem_u32(&pp->bars[st]), (pr / kStages) & 1)) {
+                atomicOr(a.err, 1);
+                vp->abort_at = pr;
+            }
+            const uint8_t* sk = ring + st * Smem<HD>::kStageBytes;
+            const uint8_t* sv = sk + Smem<HD>::kHalfBytes;
+            const int v0 = tile_valid(a, u, 2 * pr), v1 = tile_valid(a, u, 2 * pr + 1);
+            const int tbase = sp * TW;
+            // ---- scores: s[t][row] for this warp's TW tokens
+            for (int s0 = 0; s0 < TW; s0 += TPS) {
+                const int t = tbase + s0 + ts;  // token within the stage
+                const uint4 kw = *reinterpret_cast<const uint4*>(sk + t * (HD * 2) + swz(t, dg) * 16);
+                const uint32_t kk[4] = {kw.x, kw.y, kw.z, kw.w};
+                float kf[8];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    kf[2 * k] = bf_lo(kk[k]);
+                    kf[2 * k + 1] = bf_hi(kk[k]);
+                }
+                float acc[NR];
+#pragma unroll
+                for (int r = 0; r < NR; ++r) {
+                    float x = 0.f;
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) x = fmaf(qf[r][k], kf[k], x);
+                    acc[r] = x;
+                }
+                float s = transpose_reduce(acc, lane);
+                const int valid = (t & 31) < ((t < kBlockTokens) ? v0 : v1);
+                if (!valid) s = -INFINITY;
+                if (reduce_writer(lane)) sc[(s0 + ts) * NR + reduce_row(lane)] = s;
+            }
+            __syncwarp();
+            // ---- online softmax: quad r owns row r, tokens strided by 4
+            float alpha;
+            {
+                const int r = lane >> 2, q4 = lane & 3;
+                float mx = -INFINITY;
+                for (int t = q4; t < TW; t += 4) mx = fmaxf(mx, sc[t * NR + r]);
+                mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+                mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+                const float m_new = fmaxf(m_run, mx);
+                const float m_use = (m_new == -INFINITY) ? 0.f : m_new;  // all masked so far
+                alpha = fast_exp2(m_run - m_use);
+                float sum = 0.f;
+                for (int t = q4; t < TW; t += 4) {
+                    const float p = fast_exp2(sc[t * NR + r] - m_use);
+                    sc[t * NR + r] = p;
+                    sum += p;
+                }
+                sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+                sum += __shfl_xor_sync(0xffffffffu, sum, 2);
+                l_run = l_run * alpha + sum;
+                m_run = m_new;
+            }
+            __syncwarp();
+            // ---- rescale and accumulate P.V
+            if (!__all_sync(0xffffffffu, alpha == 1.f)) {
+#pragma unroll
+                for (int r = 0; r < NR; ++r) {
+                    const float al = __shfl_sync(0xffffffffu, alpha, r * 4);
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) o[r][k] *= al;
+                }
+            }
+            for (int s0 = 0; s0 < TW; s0 += TPS) {
+                const int t = tbase + s0 + ts;
+                const uint4 vw = *reinterpret_cast<const uint4*>(sv + t * (HD * 2) + swz(t, dg) * 16);
+                const uint32_t vv[4] = {vw.x, vw.y, vw.z, vw.w};
+                float vf[8];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    vf[2 * k] = bf_lo(vv[k]);
+                    vf[2 * k + 1] = bf_hi(vv[k]);
+                }
+                const float4 p0 = *reinterpret_cast<const float4*>(&sc[(s0 + ts) * NR]);
+                const float4 p1 = *reinterpret_cast<const float4*>(&sc[(s0 + ts) * NR + 4]);
+                const float p[NR] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+#pragma unroll
+                for (int r = 0; r < NR; ++r)
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) o[r][k] = fmaf(p[r], vf[k], o[r][k]);
+            }
+            __syncthreads();  // every warp is done with stage st
+            if (vp->abort_at >= 0) break;
+            if (tid == 0 && pr + kStages < n_pairs) {
+                fence_proxy_async();
+                issue_pair<HD>(a, u, ring, smem_u32(&pp->bars[st]), pr + kStages, st);
+                vp->issued = pr + kStages + 1;
+            }
+        }
+        if (vp->abort_at >= 0) return;  // copies may still land in the ring
+        // ---- fold the TPS token slots of each lane column
+#pragma unroll
+        for (int off = LPT; off < 32; off <<= 1)
+#pragma unroll
+            for (int r = 0; r < NR; ++r)
+#pragma unroll
+                for (int k = 0; k < 8; ++k) o[r][k] += __shfl_xor_sync(0xffffffffu, o[r][k], off);
+        __syncthreads();  // scratch and ring are reused below
+        // ---- combine the token splits of each row group through shared memory
+        float* cm = reinterpret_cast<float*>(ring);          // [warp][NR] max
+        float* cl = cm + 4 * NR;                             // [warp][NR] sum
+        float* co = cl + 4 * NR;                             // [warp][NR][HD]
+        if ((lane & 3) == 0) {
+            cm[warp * NR + (lane >> 2)] = m_run;
+            cl[warp * NR + (lane >> 2)] = l_run;
+        }
+        if (ts == 0) {
+#pragma unroll
+            for (int r = 0; r < NR; ++r) {
+                float4* dst = reinterpret_cast<float4*>(co + (warp * NR + r) * HD + dg * 8);
+                dst[0] = make_float4(o[r][0], o[r][1], o[r][2], o[r][3]);
+                dst[1] = make_float4(o[r][4], o[r][5], o[r][6], o[r][7]);
+            }
+        }
+        __syncthreads();
+        if (sp == 0) {
+            // this warp writes rows rg*8 .. rg*8+7; lanes: row = lane / 4, 4 lanes per row
+            const int r = lane >> 2, q4 = lane & 3;
+            const int rr = rg * NR + r;
+            float M = -INFINITY;
+            for (int s = 0; s < n_sp; ++s) M = fmaxf(M, cm[(s * n_rg + rg) * NR + r]);
+            float L = 0.f;
+            float w[4];
+            for (int s = 0; s < n_sp; ++s) {
+                const float ms = cm[(s * n_rg + rg) * NR + r];
+                w[s] = (ms == -INFINITY) ? 0.f : fast_exp2(ms - M);
+                L += w[s] * cl[(s * n_rg + rg) * NR + r];
+            }
+            if (rr < u.n_rows) {
+                const int item_row = u.row0 + rr;
+                const int slot = u.slot_base + item_row / a.group;
+                const int qh = u.kvh * a.group + item_row % a.group;
+                float* dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
+                const float inv = 1.f / L;
+                for (int d = q4 * 4; d < HD; d += 16) {
+                    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                    for (int s = 0; s < n_sp; ++s) {
+                        const float4 x = *reinterpret_cast<const float4*>(co + ((s * n_rg + rg) * NR + r) * HD + d);
+                        acc.x += w[s] * x.x;
+                        acc.y += w[s] * x.y;
+                        acc.z += w[s] * x.z;
+                        acc.w += w[s] * x.w;
+                    }
+                    *reinterpret_cast<float4*>(dst + d) = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+                }
+                if (q4 == 0) a.part_lse[(int64_t)slot * a.hq + qh] = M + __log2f(L);
+            }
+        }
+    }
+};
+
+// ---- tensor-core path: 16-row MMA tiles, one per warp -------------------
+template <int HD>
+struct TensorPath {
+    static constexpr int KS = HD / 16;  // k-steps of Q.K^T
+    static constexpr int NT = HD / 8;   // n-tiles of the output
+
+    __device__ static void run(const DecodeArgs& a, const UnitDesc& u, uint8_t* ring, Pipe* pp) {
+        volatile Pipe* vp = pp;
+        const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+        const int n_mt = (u.n_rows + 15) / 16;  // 1..4
+        const int n_sp = (n_mt == 1) ? 4 : (n_mt == 2) ? 2 : 1;
+        const int mt = warp % n_mt, sp = warp / n_mt;
+        const bool active = sp < n_sp;
+        const int TW = kStageTokens / n_sp;  // 16, 32 or 64 tokens per stage
+        const int g4 = lane >> 2, c4 = lane & 3;
+
+        // Q fragments (rows g4 and g4 + 8 of this warp's tile)
+        uint32_t qa[KS][4];
+        {
+            const uint16_t* qrow[2] = {nullptr, nullptr};
+            for (int h = 0; h < 2; ++h) {
+                const int rr = mt * 16 + g4 + 8 * h;
+                if (active && rr < u.n_rows) {
+                    const int item_row = u.row0 + rr;
+                    const int occ = a.occ[u.occ_off + item_row / a.group];
+                    const int qh = u.kvh * a.group + item_row % a.group;
+                    qrow[h] = a.q + ((int64_t)occ * a.hq + qh) * HD;
+                }
+            }
+#pragma unroll
+            for (int ks = 0; ks < KS; ++ks) {
+                const int c0 = ks * 16 + 2 * c4;
+                qa[ks][0] = qrow[0] ? *reinterpret_cast<const uint32_t*>(qrow[0] + c0) : 0u;
+                qa[ks][1] = qrow[1] ? *reinterpret_cast<const uint32_t*>(qrow[1] + c0) : 0u;
+                qa[ks][2] = qrow[0] ? *reinterpret_cast<const uint32_t*>(qrow[0] + c0 + 8) : 0u;
+                qa[ks][3] = qrow[1] ? *reinterpret_cast<const uint32_t*>(qrow[1] + c0 + 8) : 0u;
+            }
+        }
+        float o[NT][4];
+#pragma unroll
+        for (int j = 0; j < NT; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+        float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};  // rows g4, g4 + 8 (lane partial l)
+
+        const int n_pairs = (u.n_tiles + 1) / 2;
+        for (int pr = 0; pr < n_pairs; ++pr) {
+            const int st = pr % kStages;
+            if (!mbar_wait(smem_u32(&pp->bars[st]), (pr / kStages) & 1)) {
+                atomicOr(a.err, 1);
+                vp->abort_at = pr;
+            }
+            if (active) {
+                const uint32_t sk = smem_u32(ring + st * Smem<HD>::kStageBytes);
+                const uint32_t sv = sk + Smem<HD>::kHalfBytes;
+                const int v0 = tile_valid(a, u, 2 * pr), v1 = tile_valid(a, u, 2 * pr + 1);
+                const int tbase = sp * TW;
+                for (int kb = 0; kb < TW; kb += 16) {
+                    // S = Q K^T for 16 tokens: two n8 tiles
+                    float s[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+                    const int mi = lane >> 3, ri = lane & 7;
+#pragma unroll
+                    for (int ks = 0; ks < KS; ++ks) {
+                        const int tok = tbase + kb + (mi >> 1) * 8 + ri;
+                        const int ch = ks * 2 + (mi & 1);
+                        uint32_t b0, b1, b2, b3;
+                        ldsm_x4(sk + tok * (HD * 2) + swz(tok, ch) * 16, b0, b1, b2, b3);
+                        mma_bf16(s[0], qa[ks], b0, b1);
+                        mma_bf16(s[1], qa[ks], b2, b3);
+                    }
+                    // scale, mask, online softmax over these 16 tokens
+                    float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+                    for (int j = 0; j < 2; ++j)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const int tok = tbase + kb + j * 8 + 2 * c4 + (e & 1);
+                            const int lim = (tok < kBlockTokens) ? v0 : v1;
+                            const float x = ((tok & 31) < lim) ? s[j][e] * a.qk_scale_log2 : -INFINITY;
+                            s[j][e] = x;
+                            mx[e >> 1] = fmaxf(mx[e >> 1], x);
+                        }
+                    float alpha[2], m_use[2];
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], 1));
+                        mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], 2));
+                        const float m_new = fmaxf(m_run[h], mx[h]);
+                        m_use[h] = (m_new == -INFINITY) ? 0.f : m_new;
+                        alpha[h] = fast_exp2(m_run[h] - m_use[h]);
+                        m_run[h] = m_new;
+                        l_run[h] *= alpha[h];
+                    }
+                    uint32_t pa[4];
+#pragma unroll
+                    for (int j = 0; j < 2; ++j) {
+                        const float p0 = fast_exp2(s[j][0] - m_use[0]), p1 = fast_exp2(s[j][1] - m_use[0]);
+                        const float p2 = fast_exp2(s[j][2] - m_use[1]), p3 = fast_exp2(s[j][3] - m_use[1]);
+                        l_run[0] += p0 + p1;
+                        l_run[1] += p2 + p3;
+                        pa[2 * j] = pack_bf16(p0, p1);
+                        pa[2 * j + 1] = pack_bf16(p2, p3);
+                    }
+                    // A fragment of P: (row g, tok 2c..) (row g+8, tok 2c..) (row g, tok 2c+8..) (row g+8, ..)
+                    const uint32_t pfrag[4] = {pa[0], pa[1], pa[2], pa[3]};
+#pragma unroll
+                    for (int j = 0; j < NT; ++j) {
+                        o[j][0] *= alpha[0];
+                        o[j][1] *= alpha[0];
+                        o[j][2] *= alpha[1];
+                        o[j][3] *= alpha[1];
+                    }
+                    // O += P V: V^T fragments via ldmatrix.trans, two n8 tiles per load
+#pragma unroll
+                    for (int dp = 0; dp < HD / 16; ++dp) {
+                        const int tok = tbase + kb + (mi & 1) * 8 + ri;
+                        const int ch = dp * 2 + (mi >> 1);
+                        uint32_t b0, b1, b2, b3;
+                        ldsm_x4_t(sv + tok * (HD * 2) + swz(tok, ch) * 16, b0, b1, b2, b3);
+                        mma_bf16(o[2 * dp], pfrag, b0, b1);
+                        mma_bf16(o[2 * dp + 1], pfrag, b2, b3);
+                    }
+                }
+            }
+            __syncthreads();
+            if (vp->abort_at >= 0) break;
+            if (tid == 0 && pr + kStages < n_pairs) {
+                fence_proxy_async();
+                issue_pair<HD>(a, u, ring, smem_u32(&pp->bars[st]), pr + kStages, st);
+                vp->issued = pr + kStages + 1;
+            }
+        }
+        if (vp->abort_at >= 0) return;  // copies may still land in the ring
+        // full row sums over the quad
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            l_run[h] += __shfl_xor_sync(0xffffffffu, l_run[h], 1);
+            l_run[h] += __shfl_xor_sync(0xffffffffu, l_run[h], 2);
+        }
+        __syncthreads();
+        // combine token splits: warps (mt, sp>0) park (m, l, o) in shared memory
+        float* park = reinterpret_cast<float*>(ring);  // [warp][16 rows][HD + 2]
+        constexpr int PW = 16 * (HD + 2);
+        if (active && sp > 0) {
+            float* p = park + warp * PW;
+#pragma unroll
+            for (int j = 0; j < NT; ++j)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) p[(g4 + 8 * (e >> 1)) * (HD + 2) + j * 8 + 2 * c4 + (e & 1)] = o[j][e];
+            if (c4 == 0)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    p[(g4 + 8 * h) * (HD + 2) + HD] = m_run[h];
+                    p[(g4 + 8 * h) * (HD + 2) + HD + 1] = l_run[h];
+                }
+        }
+        __syncthreads();
+        if (!active || sp != 0) return;
+        for (int s = 1; s < n_sp; ++s) {
+            const float* p = park + (s * n_mt + mt) * PW;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int row = g4 + 8 * h;
+                const float ms = p[row * (HD + 2) + HD], ls = p[row * (HD + 2) + HD + 1];
+                const float M = fmaxf(m_run[h], ms);
+                const float Mu = (M == -INFINITY) ? 0.f : M;
+                const float wa = fast_exp2(m_run[h] - Mu), wb = fast_exp2(ms - Mu);
+#pragma unroll
+                for (int j = 0; j < NT; ++j) {
+                    o[j][2 * h] = o[j][2 * h] * wa + wb * p[row * (HD + 2) + j * 8 + 2 * c4];
+                    o[j][2 * h + 1] = o[j][2 * h + 1] * wa + wb * p[row * (HD + 2) + j * 8 + 2 * c4 + 1];
+                }
+                l_run[h] = l_run[h] * wa + ls * wb;
+                m_run[h] = M;
+            }
+        }
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int rr = mt * 16 + g4 + 8 * h;
+            if (rr >= u.n_rows) continue;
+            const int item_row = u.row0 + rr;
+            const int slot = u.slot_base + item_row / a.group;
+            const int qh = u.kvh * a.group + item_row % a.group;
+            float* dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
+            const float inv = 1.f / l_run[h];
+#pragma unroll
+            for (int j = 0; j < NT; ++j)
+                *reinterpret_cast<float2*>(dst + j * 8 + 2 * c4) = make_float2(o[j][2 * h] * inv, o[j][2 * h + 1] * inv);
+            if (c4 == 0) a.part_lse[(int64_t)slot * a.hq + qh] = m_run[h] + __log2f(l_run[h]);
+        }
+    }
+};
+
+template <int HD>
+__global__ void __launch_bounds__(kThreads, 2) decode_kernel(const DecodeArgs a) {
+    extern __shared__ __align__(128) uint8_t ring[];
+    __shared__ __align__(16) Pipe pipe;
+    __shared__ __align__(16) float cc_scratch[4 * kStageTokens * 8];
+    const int tid = threadIdx.x;
+
+    UnitDesc u;
+    {
+        const int* w = a.units + (int64_t)blockIdx.x * kUnitWords;
+        u.tile_off = w[U_TILE_OFF];
+        u.n_tiles = w[U_N_TILES];
+        u.occ_off = w[U_OCC_OFF];
+        u.row0 = w[U_ROW0];
+        u.n_rows = w[U_N_ROWS];
+        u.slot_base = w[U_SLOT_BASE];
+        u.kvh = w[U_KVH];
+        u.kind = w[U_KIND];
+    }
+    // zero the ring once: rows past a partial block are never copied and must
+    // hold finite values (their probabilities are exactly 0)
+    {
+        uint4* r4 = reinterpret_cast<uint4*>(ring);
+        for (int i = tid; i < Smem<HD>::kBytes / 16; i += kThreads) r4[i] = make_uint4(0, 0, 0, 0);
+    }
+    if (tid == 0) {
+        pipe.abort_at = -1;
+        for (int s = 0; s < kStages; ++s) mbar_init(smem_u32(&pipe.bars[s]), 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    fence_proxy_async();
+    __syncthreads();
+    if (tid == 0) {
+        const int n_pairs = (u.n_tiles + 1) / 2;
+        int p = 0;
+        for (; p < kStages && p < n_pairs; ++p) issue_pair<HD>(a, u, ring, smem_u32(&pipe.bars[p]), p, p);
+        pipe.issued = p;
+    }
+    if (u.kind == KIND_TENSOR)
+        TensorPath<HD>::run(a, u, ring, &pipe);
+    else
+        CudaCorePath<HD>::run(a, u, ring, &pipe, cc_scratch);
+    // After a wait ran out, let every issued copy land (each wait bounded)
+    // before the CTA exits: pairs abort_at .. issued-1 are outstanding, and
+    // each stage holds at most one of them.
+    if (tid == 0 && pipe.abort_at >= 0)
+        for (int p = pipe.abort_at; p < pipe.issued; ++p) mbar_wait(smem_u32(&pipe.bars[p % kStages]), (p / kStages) & 1);
+}
+
+// ------------------------------------------------------------------- merge --
+template <int HD>
+__global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
+    constexpr int DPL = HD / 32;  // dims per lane: 4 or 2
+    const int warp_global = blockIdx.x * 4 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (warp_global >= a.n * a.hq) return;
+    const int i = warp_global / a.hq, qh = warp_global % a.hq;
+    const int beg = a.merge_off[i], end = a.merge_off[i + 1];
+    float M = -INFINITY;
+    for (int k = beg + lane; k < end; k += 32) M = fmaxf(M, a.part_lse[(int64_t)a.merge_slot[k] * a.hq + qh]);
+#pragma unroll
+    for (int off = 16; off; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    float acc[DPL];
+#pragma unroll
+    for (int d = 0; d < DPL; ++d) acc[d] = 0.f;
+    float L = 0.f;
+    for (int k = beg; k < end; ++k) {
+        const int64_t slot = a.merge_slot[k];
+        const float w = fast_exp2(a.part_lse[slot * a.hq + qh] - M);
+        L += w;
+        const float* src = a.part_o + (slot * a.hq + qh) * HD + lane * DPL;
+        if constexpr (DPL == 4) {
+            const float4 x = *reinterpret_cast<const float4*>(src);
+            acc[0] += w * x.x;
+            acc[1] += w * x.y;
+            acc[2] += w * x.z;
+            acc[3] += w * x.w;
+        } else {
+            const float2 x = *reinterpret_cast<const float2*>(src);
+            acc[0] += w * x.x;
+            acc[1] += w * x.y;
+        }
+    }
+    const float inv = 1.f / L;
+    uint16_t* dst = a.out + ((int64_t)i * a.hq + qh) * HD + lane * DPL;
+    if constexpr (DPL == 4) {
+        const uint32_t lo = pack_bf16(acc[0] * inv, acc[1] * inv), hi = pack_bf16(acc[2] * inv, acc[3] * inv);
+        *reinterpret_cast<uint2*>(dst) = make_uint2(lo, hi);
+    } else {
+        *reinterpret_cast<uint32_t*>(dst) = pack_bf16(acc[0] * inv, acc[1] * inv);
+    }
+    if (lane == 0) a.lse[(int64_t)i * a.hq + qh] = (M + __log2f(L)) * 0.69314718055994531f;
+}
+
+template <int HD>
+cudaError_t set_decode_attrs() {
+    static cudaError_t once = cudaFuncSetAttribute(decode_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                   Smem<HD>::kBytes);
+    return once;
+}
+
+}  // namespace
+
+int decode_smem_bytes(int head_dim) { return head_dim == 64 ? Smem<64>::kBytes : Smem<128>::kBytes; }
+
+cudaError_t launch_append(int hd, const AppendArgs& a, cudaStream_t s) {
+    const int64_t chunks = 2ll * a.n_tokens * a.hkv * (hd / 8);
+    const int grid = (int)std::min<int64_t>((chunks + 255) / 256, 152 * 16);
+    if (hd == 64)
+        append_kernel<64><<<grid, 256, 0, s>>>(a);
+    else
+        append_kernel<128><<<grid, 256, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gather(int hd, const GatherArgs& a, int64_t n_tokens, cudaStream_t s) {
+    const int64_t chunks = 2ll * n_tokens * a.hkv * (hd / 8);
+    const int grid = (int)std::min<int64_t>((chunks + 255) / 256, 152 * 16);
+    if (hd == 64)
+        gather_kernel<64><<<grid, 256, 0, s>>>(a, n_tokens);
+    else
+        gather_kernel<128><<<grid, 256, 0, s>>>(a, n_tokens);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_decode(int hd, const DecodeArgs& a, cudaStream_t s) {
+    if (a.n_units == 0) return cudaSuccess;
+    cudaError_t e;
+    if (hd == 64) {
+        if ((e = set_decode_attrs<64>()) != cudaSuccess) return e;
+        decode_kernel<64><<<a.n_units, kThreads, Smem<64>::kBytes, s>>>(a);
+    } else {
+        if ((e = set_decode_attrs<128>()) != cudaSuccess) return e;
+        decode_kernel<128><<<a.n_units, kThreads, Smem<128>::kBytes, s>>>(a);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_merge(int hd, const MergeArgs& a, cudaStream_t s) {
+    const int64_t warps = (int64_t)a.n * a.hq;
+    if (warps == 0) return cudaSuccess;
+    const int grid = (int)((warps + 3) / 4);
+    if (hd == 64)
+        merge_kernel<64><<<grid, 128, 0, s>>>(a);
+    else
+        merge_kernel<128><<<grid, 128, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace tp
