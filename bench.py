@@ -44,6 +44,8 @@ def parse():
     p.add_argument("--workload", default=DEFAULT_WORKLOAD,
                    choices=["tiny", "qwen7b", "random_divergence", "wide_prefix", "no_sharing"])
     p.add_argument("--seed", type=int, default=0)
+    p.add_argument("--prompts", type=int, default=None,
+                   help="scale the workload down to this many prompts (small cases for ncu captures)")
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--flags", type=int, default=0, help="tp_decode_ex flags for the timed steps")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -79,6 +81,14 @@ def describe(script):
         "lse_bytes": len(script.leaves) * h.num_q_heads * 4,
         "flops": sum(per_leaf) * 4 * h.num_q_heads * h.head_dim,
     }
+
+
+def make_script(args, seed):
+    import workloads
+    kw = {"seed": seed}
+    if args.prompts is not None:
+        kw["n_seqs" if args.workload == "no_sharing" else "n_prompts"] = args.prompts
+    return workloads.by_name(args.workload, **kw)
 
 
 def workload_label(script):
@@ -223,8 +233,7 @@ def run_reference(args, rank, world):
     """--impl reference: the CPU oracle on the host cores, same metric/config."""
     if rank != 0:
         return
-    import workloads
-    script = workloads.by_name(args.workload, seed=args.seed)
+    script = make_script(args, args.seed)
     desc = describe(script)
     # each step: a bounded sample sized so warmup + steps take a few minutes
     per_step_budget = max(1.0, 150.0 / max(1, args.steps + args.warmup))
@@ -278,7 +287,7 @@ def main():
     if world > 1:
         dist.barrier()
 
-    script = workloads.by_name(args.workload, seed=args.seed + rank)
+    script = make_script(args, args.seed + rank)
     desc = describe(script)
     h = script.heads
     t_setup = time.perf_counter()

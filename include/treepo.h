@@ -150,10 +150,11 @@ tp_status tp_decode(tp_tree* tree, const tp_node* leaves, int32_t n, const void*
                     float* LSE);
 
 /* tp_decode with options (bit flags below). */
-#define TP_DECODE_NO_SHARE 1u        /* schedule every leaf's whole path on its own  */
-#define TP_DECODE_SMALL_ON_TENSOR 2u /* groups of < 16 query rows on the tensor-core */
-                                     /* kernel too (default: CUDA-core kernel)       */
-#define TP_DECODE_NO_CACHE 4u        /* rebuild the schedule even if cached          */
+#define TP_DECODE_NO_SHARE 1u         /* schedule every leaf's whole path on its own */
+#define TP_DECODE_CUDA_CORE_SMALL 2u  /* units of < 16 query rows on the CUDA-core   */
+                                      /* path (default: tensor cores, rows padded to */
+                                      /* one 16-row MMA tile)                        */
+#define TP_DECODE_NO_CACHE 4u         /* rebuild the schedule even if cached         */
 tp_status tp_decode_ex(tp_tree* tree, const tp_node* leaves, int32_t n, const void* Q, void* O,
                        float* LSE, uint32_t flags);
 

@@ -23,7 +23,7 @@ __all__ = [
     "tp_set_stream", "tp_add_root", "tp_append_segment", "tp_fork", "tp_prune", "tp_decode", "tp_decode_ex",
     "tp_sync", "tp_last_error", "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop",
     "tp_debug_path", "tp_debug_gather",
-    "tp_debug_schedule", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_SMALL_ON_TENSOR", "TP_DECODE_NO_CACHE",
+    "tp_debug_schedule", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE",
     "EXPORTED_SYMBOLS",
 ]
 
@@ -32,7 +32,7 @@ _LIB_PATH = os.path.join(_HERE, "libtreepo.so")
 _lib: Optional[ctypes.CDLL] = None
 
 TP_DECODE_NO_SHARE = 1
-TP_DECODE_SMALL_ON_TENSOR = 2
+TP_DECODE_CUDA_CORE_SMALL = 2
 TP_DECODE_NO_CACHE = 4
 
 STATUS_NAMES = {0: "OK", -1: "INVALID_ARG", -2: "OOM", -3: "BAD_NODE", -4: "FROZEN", -5: "NOT_LEAF",

@@ -106,7 +106,7 @@ constexpr int32_t kMaxChunkTiles = 32;
 tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t flags, Schedule& S) {
     const int32_t hq = t->cfg.num_q_heads, hkv = t->cfg.num_kv_heads, g = hq / hkv;
     const bool share = !(flags & TP_DECODE_NO_SHARE);
-    const bool small_on_tensor = (flags & TP_DECODE_SMALL_ON_TENSOR) != 0;
+    const bool cuda_core_small = (flags & TP_DECODE_CUDA_CORE_SMALL) != 0;
     for (int32_t i = 0; i < n; ++i) {
         tp_status st = check_live(t, leaves[i], true);
         if (st != TP_OK) return st;
@@ -186,10 +186,15 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
         }
     }
 
-    // 4. chunk size: enough units to fill the GPU several times over
+    // 4. chunk size: enough units to fill the GPU several times over, but
+    //    every chunk of an item costs one fp32 partial per stacked row
+    //    ((head_dim + 1) * 4 bytes written, then read by the merge); an item
+    //    with R rows per kv head is cut no finer than 1.25 R blocks, which
+    //    keeps that traffic under ~5% of the chunk's KV bytes.
     int64_t work = 0;
     for (const Item& it : items) work += (int64_t)it.n_tiles * hkv;
-    int32_t chunk = (int32_t)std::min<int64_t>(kMaxChunkTiles, std::max<int64_t>(kMinChunkTiles, (work + kTargetUnits - 1) / kTargetUnits));
+    const int32_t chunk = (int32_t)std::min<int64_t>(
+        kMaxChunkTiles, std::max<int64_t>(kMinChunkTiles, (work + kTargetUnits - 1) / kTargetUnits));
 
     // 5. units, partial slots and merge entries
     std::vector<int32_t> tensor_units, small_units;
@@ -197,7 +202,9 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     int32_t n_slots = 0;
     for (const Item& it : items) {
         if (it.n_tiles == 0) continue;
-        const int32_t n_chunks = (it.n_tiles + chunk - 1) / chunk;
+        const int32_t rows_chunk = (it.n_occ * g * 5 + 3) / 4;
+        const int32_t n_chunks = rows_chunk > chunk ? std::max(1, it.n_tiles / rows_chunk)
+                                                    : (it.n_tiles + chunk - 1) / chunk;
         const int32_t base = it.n_tiles / n_chunks, extra = it.n_tiles % n_chunks;
         const int32_t rows = it.n_occ * g;
         int32_t toff = it.tile_off;
@@ -210,7 +217,7 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
                 pair_slot.push_back(slot_base + p);
             }
             for (int32_t h = 0; h < hkv; ++h) {
-                if (rows < kTensorMinRows && !small_on_tensor) {
+                if (rows < kTensorMinRows && cuda_core_small) {
                     const int32_t u[kUnitWords] = {toff, nt, it.occ_off, 0, rows, slot_base, h, KIND_CUDA_CORE};
                     small_units.insert(small_units.end(), u, u + kUnitWords);
                 } else {

@@ -21,7 +21,8 @@ enum UnitWord { U_TILE_OFF, U_N_TILES, U_OCC_OFF, U_ROW0, U_N_ROWS, U_SLOT_BASE,
 enum UnitKind { KIND_CUDA_CORE = 0, KIND_TENSOR = 1 };
 constexpr int kSchedHeaderWords = 16;
 constexpr int32_t kSchedMagic = 0x54505344;
-// Query rows at or above which a unit runs on the tensor-core path.
+// Units with fewer query rows may run on the CUDA-core path
+// (TP_DECODE_CUDA_CORE_SMALL); every other unit runs on tensor cores.
 constexpr int kTensorMinRows = 16;
 // Query rows per tensor-core unit (4 warps x one 16-row MMA tile each).
 constexpr int kTensorRowsPerUnit = 64;

@@ -267,10 +267,10 @@ def check_schedule(f, ids, model, script, leaves_sid, flags=0):
         toff, nt, ooff, row0, nrows, sbase, kvh, kind = (int(x) for x in u)
         assert 0 <= kvh < heads.num_kv_heads
         if kind == 0:
-            assert nrows < 16
+            assert nrows < 16 and flags & tp.TP_DECODE_CUDA_CORE_SMALL
         else:
             assert 1 <= nrows <= 64
-            if not flags & tp.TP_DECODE_SMALL_ON_TENSOR:
+            if flags & tp.TP_DECODE_CUDA_CORE_SMALL:
                 assert nrows >= 16 or row0 > 0
         tok = _expand(S["tiles"][toff:toff + nt])
         assert len(tok) > 0
@@ -296,7 +296,7 @@ def check_schedule(f, ids, model, script, leaves_sid, flags=0):
 
 
 @pytest.mark.parametrize("seed", range(6))
-@pytest.mark.parametrize("flags", [0, tp.TP_DECODE_NO_SHARE, tp.TP_DECODE_SMALL_ON_TENSOR])
+@pytest.mark.parametrize("flags", [0, tp.TP_DECODE_NO_SHARE, tp.TP_DECODE_CUDA_CORE_SMALL])
 def test_schedule_covers_every_path_token_once(seed, flags):
     s = workloads.random_tree(seed=seed, n_prompts=3, max_depth=5, prompt_range=(1, 300), seg_range=(1, 150),
                               heads=workloads.Heads(8, 2, 64))
@@ -321,6 +321,18 @@ def test_schedule_on_named_workloads(name, kw):
         uniq_blocks |= {x // BT for x in m.path_slots(lf).tolist()}
     read = sum(int(u[1]) for u in S["units"] if int(u[3]) == 0)
     assert read == len(uniq_blocks) * s.heads.num_kv_heads
+
+
+def test_long_shared_node_is_cut_into_chunks():
+    s = workloads.shared_prompt()
+    f = meta_forest(heads=s.heads, pool_blocks=1 << 10)
+    ids = f.replay(s.ops)
+    m = oracle.OracleForest(block_tokens=BT, pool_blocks=1 << 10).replay(s)
+    S = check_schedule(f, ids, m, s, s.leaves)
+    # 63 prompt blocks, 24 rows per kv head: chunks of >= 30 blocks
+    prompt_units = [u for u in S["units"] if int(u[1]) > 10]
+    assert len({int(u[0]) for u in prompt_units}) >= 2
+    assert all(int(u[1]) >= 30 for u in prompt_units)
 
 
 def test_schedule_without_sharing_reads_every_path():

@@ -35,7 +35,7 @@ import torch
 
 __all__ = [
     "Heads", "Script", "tiny", "qwen7b", "random_divergence", "wide_prefix",
-    "no_sharing", "random_tree", "single_path", "by_name", "CONFIG_NAMES",
+    "no_sharing", "random_tree", "single_path", "shared_prompt", "by_name", "CONFIG_NAMES",
 ]
 
 
@@ -353,6 +353,20 @@ def random_tree(seed: int = 0, heads: Heads = Heads(8, 2, 64), n_prompts: int = 
     if leaves:
         leaves.append(leaves[0])
     return Script("random_tree", heads, seed, b.ops, leaves, b.kv_len, "irregular forest")
+
+
+def shared_prompt(seed: int = 0, prompt: int = 2000, n_leaves: int = 3, leaf_tokens: Sequence[int] = (40, 7, 90),
+                  heads: Heads = Heads(16, 2, 128)) -> Script:
+    """One long prompt forked into a few short leaves (long shared node with
+    few stacked rows)."""
+    b = _Builder()
+    r = b.root()
+    b.append(r, prompt)
+    kids = b.fork(r, n_leaves)
+    for c, n in zip(kids, leaf_tokens):
+        b.append(c, n)
+    return Script("shared_prompt", heads, seed, b.ops, kids, b.kv_len,
+                  f"prompt {prompt} shared by {n_leaves} leaves")
 
 
 CONFIG_NAMES = ("tiny", "qwen7b", "random_divergence", "wide_prefix", "no_sharing")
