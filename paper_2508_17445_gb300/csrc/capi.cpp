@@ -129,8 +129,8 @@ tp_status tp_tree_create(const tp_config* cfg, tp_tree** out) {
     t->stream = (cudaStream_t)cfg->cuda_stream;
     t->pool.init(cfg->pool_blocks);
     if (cfg->pool) {
-        cudaError_t e = cudaMalloc((void**)&t->d_err, sizeof(int32_t));
-        if (e == cudaSuccess) e = cudaMemsetAsync(t->d_err, 0, sizeof(int32_t), t->stream);
+        cudaError_t e = cudaMalloc((void**)&t->d_err, 4 * sizeof(int32_t));
+        if (e == cudaSuccess) e = cudaMemsetAsync(t->d_err, 0, 4 * sizeof(int32_t), t->stream);
         if (e != cudaSuccess) {
             g_create_err = std::string("device error flag: ") + cudaGetErrorString(e);
             cudaGetLastError();
@@ -316,6 +316,10 @@ tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void*
     a.part_o = t->d_part;
     a.part_lse = t->d_part + (int64_t)S.n_slots * hq * hd;
     a.err = t->d_err;
+    a.counters = t->d_err + 1;
+    a.counter = nullptr;
+    a.n_tensor_units = S.n_tensor;
+    a.unit_begin = a.unit_end = 0;
     a.head_bytes = t->cfg.block_tokens * hd * 2;
     a.block_bytes = (int64_t)2 * t->cfg.num_kv_heads * a.head_bytes;
     a.n_units = S.n_units;
@@ -337,6 +341,7 @@ tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void*
     m.part_lse = a.part_lse;
     m.out = (uint16_t*)O;
     m.lse = LSE;
+    m.counters = t->d_err + 1;
     m.n = n;
     m.hq = hq;
     {

@@ -41,6 +41,10 @@ struct DecodeArgs {
     float* part_o;      // [slot][Hq][hd], normalised partial output
     float* part_lse;    // [slot][Hq], log2-domain partial LSE
     int32_t* err;
+    int32_t* counters;    // [2] next unit per kind (0 at launch; the merge re-arms them)
+    int32_t* counter;     // the counter of the launch in flight (set by the launcher)
+    int32_t n_tensor_units;  // units [0, n_tensor_units) are tensor units
+    int32_t unit_begin, unit_end;  // unit range of the launch in flight
     int64_t block_bytes;  // bytes of one pool block (K and V, all kv heads)
     int32_t head_bytes;   // bytes of one (block, K|V, kv head) tile
     int32_t n_units;
@@ -57,6 +61,7 @@ struct MergeArgs {
     const float* part_lse;
     uint16_t* out;  // bf16 [n][Hq][hd]
     float* lse;     // [n][Hq], natural log
+    int32_t* counters;  // decode's two unit counters, reset to 0 here
     int32_t n;
     int32_t hq;
 };
@@ -140,7 +145,7 @@ struct tp_tree {
     uint32_t epoch = 0;
 
     // device scratch owned by the library
-    int32_t* d_err = nullptr;
+    int32_t* d_err = nullptr;  // [0] device error flag, [1..2] decode unit counters
     int32_t* d_sched = nullptr;
     int64_t d_sched_cap = 0;  // words
     float* d_part = nullptr;  // partial o then partial lse

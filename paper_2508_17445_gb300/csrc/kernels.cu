@@ -35,10 +35,11 @@
 namespace tp {
 namespace {
 
-constexpr int kThreads = 128;      // 4 warps per CTA
+constexpr int kConsumerWarps = 4;                          // attention warps per CTA
+constexpr int kDecodeThreads = (kConsumerWarps + 1) * 32;  // + one producer warp
 constexpr int kBlockTokens = 32;   // tokens per pool block (= tile)
 constexpr int kStageTokens = 64;   // two tiles per pipeline stage
-constexpr int kStages = 3;         // stages in the shared-memory ring
+constexpr int kStages = 2;         // stages in each CTA's shared-memory ring
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // bounded mbarrier waits: 2 s
 
 // ------------------------------------------------------------ PTX helpers --
@@ -182,56 +183,127 @@ __global__ void gather_kernel(const GatherArgs a, int64_t n_tokens) {
 }
 
 // ------------------------------------------------------------------ decode --
+// Persistent, warp-specialised kernel. Each CTA (two per SM) runs one
+// producer warp and kConsumerWarps consumer warps until the global unit
+// counter runs past the unit list (units are sorted longest first, so the
+// counter hands them out in LPT order). The producer's lane 0 fetches a unit,
+// publishes it in one of two unit slots, and streams the unit's tile pairs
+// into a ring of shared-memory stages with TMA bulk copies; it runs ahead
+// across unit boundaries, so HBM keeps streaming while the consumers finish a
+// unit (the split combine and partial stores). Every wait is an mbarrier wait
+// bounded in time; a wait that runs out sets the device error flag and the
+// kernel carries on to a bounded exit.
 struct UnitDesc {
     int tile_off, n_tiles, occ_off, row0, n_rows, slot_base, kvh, kind;
 };
+
+__device__ __forceinline__ UnitDesc load_unit(const DecodeArgs& a, int u) {
+    const int* w = a.units + (int64_t)u * kUnitWords;
+    UnitDesc d;
+    d.tile_off = w[U_TILE_OFF];
+    d.n_tiles = w[U_N_TILES];
+    d.occ_off = w[U_OCC_OFF];
+    d.row0 = w[U_ROW0];
+    d.n_rows = w[U_N_ROWS];
+    d.slot_base = w[U_SLOT_BASE];
+    d.kvh = w[U_KVH];
+    d.kind = w[U_KIND];
+    return d;
+}
 
 template <int HD>
 struct Smem {
     static constexpr int kRowBytes = HD * 2;
     static constexpr int kHalfBytes = kStageTokens * kRowBytes;  // K or V of one stage
     static constexpr int kStageBytes = 2 * kHalfBytes;
-    static constexpr int kBytes = kStages * kStageBytes;
+    static constexpr int kRingBytes = kStages * kStageBytes;
+    // split combine: kConsumerWarps x 16 rows x (HD + 2) floats; the CUDA-core
+    // combine (4 x 8 rows x HD + 64 floats) fits in the same region
+    static constexpr int kParkFloats = kConsumerWarps * 16 * (HD + 2);
+    static constexpr int kBytes = kRingBytes + kParkFloats * 4;
 };
 
-// Shared pipeline bookkeeping of one CTA.
-struct Pipe {
-    uint64_t bars[kStages];  // "stage full" barriers (transaction counted)
-    int issued;              // tile pairs issued so far (written by thread 0)
-    int abort_at;            // first pair whose wait ran out, or -1
+// Shared control block of one CTA.
+struct Ctl {
+    uint64_t full[kStages];   // stage filled (producer arrival + TMA bytes)
+    uint64_t empty[kStages];  // stage consumed (one arrival per consumer warp)
+    uint64_t ufull[2];        // unit slot published
+    uint64_t uempty[2];       // unit slot read by every consumer warp
+    uint64_t csync;           // consumer-only barrier (split combine)
+    int valid[kStages][2];    // valid tokens of the stage's two tiles (0: no tile)
+    int unit[2];
+    int abort;
 };
 
-// Producer: issue the bulk copies of tile pair `pair` into stage `st`.
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void note_timeout(const DecodeArgs& a, Ctl& c, int code) {
+    atomicOr(a.err, code);
+    *reinterpret_cast<volatile int*>(&c.abort) = 1;
+}
+
+// Producer: issue the bulk copies of one tile pair (tile words w[0..1],
+// w = -1 for a missing second tile) into stage `st`, and record the pair's
+// valid token counts for the consumers.
 template <int HD>
-__device__ __forceinline__ void issue_pair(const DecodeArgs& a, const UnitDesc& u, uint8_t* ring, uint32_t bar,
-                                           int pair, int st) {
+__device__ __forceinline__ void issue_pair(const DecodeArgs& a, Ctl& c, int kvh, uint8_t* ring, const int32_t (&w)[2],
+                                           int st) {
     constexpr int RB = HD * 2;
     uint8_t* sk = ring + st * Smem<HD>::kStageBytes;
     uint8_t* sv = sk + Smem<HD>::kHalfBytes;
+    const uint32_t bar = smem_u32(&c.full[st]);
+    int valid[2] = {0, 0};
     uint32_t bytes = 0;
-    int32_t w[2];
-    int nt = 0;
-    for (int j = 0; j < 2; ++j) {
-        const int t = 2 * pair + j;
-        if (t < u.n_tiles) {
-            w[j] = a.tiles[u.tile_off + t];
-            bytes += 2u * (uint32_t)(((w[j] & ((1 << kTileValidBits) - 1)) + 1) * RB);
-            nt = j + 1;
+    for (int j = 0; j < 2; ++j)
+        if (w[j] >= 0) {
+            valid[j] = (w[j] & ((1 << kTileValidBits) - 1)) + 1;
+            bytes += 2u * (uint32_t)(valid[j] * RB);
         }
-    }
-    mbar_arrive_expect_tx(bar, bytes);
-    for (int j = 0; j < nt; ++j) {
-        const int valid = (w[j] & ((1 << kTileValidBits) - 1)) + 1;
+    c.valid[st][0] = valid[0];
+    c.valid[st][1] = valid[1];
+    mbar_arrive_expect_tx(bar, bytes);  // release: the valid counts are visible to the stage's waiters
+    for (int j = 0; j < 2; ++j) {
+        if (!valid[j]) continue;
         const int64_t blk = w[j] >> kTileValidBits;
-        const uint8_t* src = a.pool + blk * a.block_bytes + (int64_t)u.kvh * a.head_bytes;
-        bulk_g2s(smem_u32(sk + j * kBlockTokens * RB), src, valid * RB, bar);
-        bulk_g2s(smem_u32(sv + j * kBlockTokens * RB), src + (int64_t)a.hkv * a.head_bytes, valid * RB, bar);
+        const uint8_t* src = a.pool + blk * a.block_bytes + (int64_t)kvh * a.head_bytes;
+        bulk_g2s(smem_u32(sk + j * kBlockTokens * RB), src, valid[j] * RB, bar);
+        bulk_g2s(smem_u32(sv + j * kBlockTokens * RB), src + (int64_t)a.hkv * a.head_bytes, valid[j] * RB, bar);
     }
 }
 
-__device__ __forceinline__ int tile_valid(const DecodeArgs& a, const UnitDesc& u, int t) {
-    return t < u.n_tiles ? (a.tiles[u.tile_off + t] & ((1 << kTileValidBits) - 1)) + 1 : 0;
-}
+// Consumer side of the stage ring (one instance per consumer warp).
+struct RingReader {
+    Ctl* c;
+    uint8_t* ring;
+    int stage;
+    uint32_t phase;
+    uint32_t sync_phase;
+
+    template <int HD>
+    __device__ __forceinline__ const uint8_t* acquire(const DecodeArgs& a, int& v0, int& v1) {
+        if (!mbar_wait(smem_u32(&c->full[stage]), phase)) note_timeout(a, *c, 1);
+        v0 = c->valid[stage][0];
+        v1 = c->valid[stage][1];
+        return ring + stage * Smem<HD>::kStageBytes;
+    }
+    __device__ __forceinline__ void release(int lane) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&c->empty[stage]));
+        if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+        }
+    }
+    // barrier of the consumer warps only (the producer never takes part)
+    __device__ __forceinline__ void consumers_sync(const DecodeArgs& a, int lane) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&c->csync));
+        if (!mbar_wait(smem_u32(&c->csync), sync_phase)) note_timeout(a, *c, 4);
+        sync_phase ^= 1;
+    }
+};
 
 // ---- CUDA-core path: <= 16 rows, 8 rows per warp ------------------------
 // Lane layout: LPT = HD/8 lanes share one token (8 dims each, one 16-byte
@@ -292,11 +364,11 @@ struct CudaCorePath {
     __device__ __forceinline__ static int reduce_row(int lane) { return LPT == 16 ? (lane >> 1) & 7 : lane & 7; }
     __device__ __forceinline__ static bool reduce_writer(int lane) { return LPT == 16 ? (lane & 1) == 0 : true; }
 
-    __device__ static void run(const DecodeArgs& a, const UnitDesc& u, uint8_t* ring, Pipe* pp, float* scratch) {
-        volatile Pipe* vp = pp;
-        const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    __device__ static void unit(const DecodeArgs& a, const UnitDesc& u, RingReader& rr, float* park,
+                                float* scratch) {
+        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
         const int n_rg = (u.n_rows + NR - 1) / NR;  // 1 or 2 row groups
-        const int n_sp = 4 / n_rg;                  // token splits
+        const int n_sp = kConsumerWarps / n_rg;     // token splits
         const int rg = warp % n_rg, sp = warp / n_rg;
         const int TW = kStageTokens / n_sp;  // tokens of a stage this warp handles
         const int dg = lane % LPT, ts = lane / LPT;
@@ -305,9 +377,9 @@ struct CudaCorePath {
         float qf[NR][8];
 #pragma unroll
         for (int r = 0; r < NR; ++r) {
-            const int rr = rg * NR + r;
-            if (rr < u.n_rows) {
-                const int item_row = u.row0 + rr;
+            const int rr_ = rg * NR + r;
+            if (rr_ < u.n_rows) {
+                const int item_row = u.row0 + rr_;
                 const int occ = a.occ[u.occ_off + item_row / a.group];
                 const int qh = u.kvh * a.group + item_row % a.group;
                 const uint4 w = *reinterpret_cast<const uint4*>(a.q + ((int64_t)occ * a.hq + qh) * HD + dg * 8);
@@ -333,14 +405,9 @@ struct CudaCorePath {
 
         const int n_pairs = (u.n_tiles + 1) / 2;
         for (int pr = 0; pr < n_pairs; ++pr) {
-            const int st = pr % kStages;
-            if (!mbar_wait(smem_u32(&pp->bars[st]), (pr / kStages) & 1)) {
-                atomicOr(a.err, 1);
-                vp->abort_at = pr;
-            }
-            const uint8_t* sk = ring + st * Smem<HD>::kStageBytes;
+            int v0, v1;
+            const uint8_t* sk = rr.acquire<HD>(a, v0, v1);
             const uint8_t* sv = sk + Smem<HD>::kHalfBytes;
-            const int v0 = tile_valid(a, u, 2 * pr), v1 = tile_valid(a, u, 2 * pr + 1);
             const int tbase = sp * TW;
             // ---- scores: s[t][row] for this warp's TW tokens
             for (int s0 = 0; s0 < TW; s0 += TPS) {
@@ -417,15 +484,9 @@ struct CudaCorePath {
 #pragma unroll
                     for (int k = 0; k < 8; ++k) o[r][k] = fmaf(p[r], vf[k], o[r][k]);
             }
-            __syncthreads();  // every warp is done with stage st
-            if (vp->abort_at >= 0) break;
-            if (tid == 0 && pr + kStages < n_pairs) {
-                fence_proxy_async();
-                issue_pair<HD>(a, u, ring, smem_u32(&pp->bars[st]), pr + kStages, st);
-                vp->issued = pr + kStages + 1;
-            }
+            __syncwarp();  // sc is rewritten by the next stage's scores
+            rr.release(lane);
         }
-        if (vp->abort_at >= 0) return;  // copies may still land in the ring
         // ---- fold the TPS token slots of each lane column
 #pragma unroll
         for (int off = LPT; off < 32; off <<= 1)
@@ -433,11 +494,11 @@ struct CudaCorePath {
             for (int r = 0; r < NR; ++r)
 #pragma unroll
                 for (int k = 0; k < 8; ++k) o[r][k] += __shfl_xor_sync(0xffffffffu, o[r][k], off);
-        __syncthreads();  // scratch and ring are reused below
         // ---- combine the token splits of each row group through shared memory
-        float* cm = reinterpret_cast<float*>(ring);          // [warp][NR] max
-        float* cl = cm + 4 * NR;                             // [warp][NR] sum
-        float* co = cl + 4 * NR;                             // [warp][NR][HD]
+        float* cm = park;                 // [warp][NR] max
+        float* cl = cm + 4 * NR;          // [warp][NR] sum
+        float* co = cl + 4 * NR;          // [warp][NR][HD]
+        rr.consumers_sync(a, lane);       // the previous unit's combine is done with the park
         if ((lane & 3) == 0) {
             cm[warp * NR + (lane >> 2)] = m_run;
             cl[warp * NR + (lane >> 2)] = l_run;
@@ -450,39 +511,38 @@ struct CudaCorePath {
                 dst[1] = make_float4(o[r][4], o[r][5], o[r][6], o[r][7]);
             }
         }
-        __syncthreads();
-        if (sp == 0) {
-            // this warp writes rows rg*8 .. rg*8+7; lanes: row = lane / 4, 4 lanes per row
-            const int r = lane >> 2, q4 = lane & 3;
-            const int rr = rg * NR + r;
-            float M = -INFINITY;
-            for (int s = 0; s < n_sp; ++s) M = fmaxf(M, cm[(s * n_rg + rg) * NR + r]);
-            float L = 0.f;
-            float w[4];
-            for (int s = 0; s < n_sp; ++s) {
-                const float ms = cm[(s * n_rg + rg) * NR + r];
-                w[s] = (ms == -INFINITY) ? 0.f : fast_exp2(ms - M);
-                L += w[s] * cl[(s * n_rg + rg) * NR + r];
-            }
-            if (rr < u.n_rows) {
-                const int item_row = u.row0 + rr;
-                const int slot = u.slot_base + item_row / a.group;
-                const int qh = u.kvh * a.group + item_row % a.group;
-                float* dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
-                const float inv = 1.f / L;
-                for (int d = q4 * 4; d < HD; d += 16) {
-                    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-                    for (int s = 0; s < n_sp; ++s) {
-                        const float4 x = *reinterpret_cast<const float4*>(co + ((s * n_rg + rg) * NR + r) * HD + d);
-                        acc.x += w[s] * x.x;
-                        acc.y += w[s] * x.y;
-                        acc.z += w[s] * x.z;
-                        acc.w += w[s] * x.w;
-                    }
-                    *reinterpret_cast<float4*>(dst + d) = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+        rr.consumers_sync(a, lane);
+        if (sp != 0) return;
+        // this warp writes rows rg*8 .. rg*8+7; lanes: row = lane / 4, 4 lanes per row
+        const int r = lane >> 2, q4 = lane & 3;
+        const int rr_ = rg * NR + r;
+        float M = -INFINITY;
+        for (int s = 0; s < n_sp; ++s) M = fmaxf(M, cm[(s * n_rg + rg) * NR + r]);
+        float L = 0.f;
+        float w[kConsumerWarps];
+        for (int s = 0; s < n_sp; ++s) {
+            const float ms = cm[(s * n_rg + rg) * NR + r];
+            w[s] = (ms == -INFINITY) ? 0.f : fast_exp2(ms - M);
+            L += w[s] * cl[(s * n_rg + rg) * NR + r];
+        }
+        if (rr_ < u.n_rows) {
+            const int item_row = u.row0 + rr_;
+            const int slot = u.slot_base + item_row / a.group;
+            const int qh = u.kvh * a.group + item_row % a.group;
+            float* dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
+            const float inv = 1.f / L;
+            for (int d = q4 * 4; d < HD; d += 16) {
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int s = 0; s < n_sp; ++s) {
+                    const float4 x = *reinterpret_cast<const float4*>(co + ((s * n_rg + rg) * NR + r) * HD + d);
+                    acc.x += w[s] * x.x;
+                    acc.y += w[s] * x.y;
+                    acc.z += w[s] * x.z;
+                    acc.w += w[s] * x.w;
                 }
-                if (q4 == 0) a.part_lse[(int64_t)slot * a.hq + qh] = M + __log2f(L);
+                *reinterpret_cast<float4*>(dst + d) = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
             }
+            if (q4 == 0) a.part_lse[(int64_t)slot * a.hq + qh] = M + __log2f(L);
         }
     }
 };
@@ -493,9 +553,8 @@ struct TensorPath {
     static constexpr int KS = HD / 16;  // k-steps of Q.K^T
     static constexpr int NT = HD / 8;   // n-tiles of the output
 
-    __device__ static void run(const DecodeArgs& a, const UnitDesc& u, uint8_t* ring, Pipe* pp) {
-        volatile Pipe* vp = pp;
-        const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    __device__ static void unit(const DecodeArgs& a, const UnitDesc& u, RingReader& rr, float* park) {
+        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
         const int n_mt = (u.n_rows + 15) / 16;  // 1..4
         const int n_sp = (n_mt == 1) ? 4 : (n_mt == 2) ? 2 : 1;
         const int mt = warp % n_mt, sp = warp / n_mt;
@@ -508,9 +567,9 @@ struct TensorPath {
         {
             const uint16_t* qrow[2] = {nullptr, nullptr};
             for (int h = 0; h < 2; ++h) {
-                const int rr = mt * 16 + g4 + 8 * h;
-                if (active && rr < u.n_rows) {
-                    const int item_row = u.row0 + rr;
+                const int r = mt * 16 + g4 + 8 * h;
+                if (active && r < u.n_rows) {
+                    const int item_row = u.row0 + r;
                     const int occ = a.occ[u.occ_off + item_row / a.group];
                     const int qh = u.kvh * a.group + item_row % a.group;
                     qrow[h] = a.q + ((int64_t)occ * a.hq + qh) * HD;
@@ -532,15 +591,11 @@ struct TensorPath {
 
         const int n_pairs = (u.n_tiles + 1) / 2;
         for (int pr = 0; pr < n_pairs; ++pr) {
-            const int st = pr % kStages;
-            if (!mbar_wait(smem_u32(&pp->bars[st]), (pr / kStages) & 1)) {
-                atomicOr(a.err, 1);
-                vp->abort_at = pr;
-            }
+            int v0, v1;
+            const uint8_t* stage = rr.acquire<HD>(a, v0, v1);
             if (active) {
-                const uint32_t sk = smem_u32(ring + st * Smem<HD>::kStageBytes);
+                const uint32_t sk = smem_u32(stage);
                 const uint32_t sv = sk + Smem<HD>::kHalfBytes;
-                const int v0 = tile_valid(a, u, 2 * pr), v1 = tile_valid(a, u, 2 * pr + 1);
                 const int tbase = sp * TW;
                 for (int kb = 0; kb < TW; kb += 16) {
                     // S = Q K^T for 16 tokens: two n8 tiles
@@ -578,6 +633,7 @@ struct TensorPath {
                         m_run[h] = m_new;
                         l_run[h] *= alpha[h];
                     }
+                    // A fragment of P: (row g, tok 2c..) (row g+8, tok 2c..) (row g, tok 2c+8..) (row g+8, ..)
                     uint32_t pa[4];
 #pragma unroll
                     for (int j = 0; j < 2; ++j) {
@@ -588,8 +644,6 @@ struct TensorPath {
                         pa[2 * j] = pack_bf16(p0, p1);
                         pa[2 * j + 1] = pack_bf16(p2, p3);
                     }
-                    // A fragment of P: (row g, tok 2c..) (row g+8, tok 2c..) (row g, tok 2c+8..) (row g+8, ..)
-                    const uint32_t pfrag[4] = {pa[0], pa[1], pa[2], pa[3]};
 #pragma unroll
                     for (int j = 0; j < NT; ++j) {
                         o[j][0] *= alpha[0];
@@ -604,68 +658,64 @@ struct TensorPath {
                         const int ch = dp * 2 + (mi >> 1);
                         uint32_t b0, b1, b2, b3;
                         ldsm_x4_t(sv + tok * (HD * 2) + swz(tok, ch) * 16, b0, b1, b2, b3);
-                        mma_bf16(o[2 * dp], pfrag, b0, b1);
-                        mma_bf16(o[2 * dp + 1], pfrag, b2, b3);
+                        mma_bf16(o[2 * dp], pa, b0, b1);
+                        mma_bf16(o[2 * dp + 1], pa, b2, b3);
                     }
                 }
             }
-            __syncthreads();
-            if (vp->abort_at >= 0) break;
-            if (tid == 0 && pr + kStages < n_pairs) {
-                fence_proxy_async();
-                issue_pair<HD>(a, u, ring, smem_u32(&pp->bars[st]), pr + kStages, st);
-                vp->issued = pr + kStages + 1;
-            }
+            rr.release(lane);
         }
-        if (vp->abort_at >= 0) return;  // copies may still land in the ring
         // full row sums over the quad
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
             l_run[h] += __shfl_xor_sync(0xffffffffu, l_run[h], 1);
             l_run[h] += __shfl_xor_sync(0xffffffffu, l_run[h], 2);
         }
-        __syncthreads();
-        // combine token splits: warps (mt, sp>0) park (m, l, o) in shared memory
-        float* park = reinterpret_cast<float*>(ring);  // [warp][16 rows][HD + 2]
-        constexpr int PW = 16 * (HD + 2);
-        if (active && sp > 0) {
-            float* p = park + warp * PW;
+        if (n_sp > 1) {
+            // token splits of one M-tile meet in shared memory: [warp][16 rows][HD + 2]
+            constexpr int PW = 16 * (HD + 2);
+            rr.consumers_sync(a, lane);  // the previous unit's combine is done with the park
+            if (active && sp > 0) {
+                float* p = park + warp * PW;
 #pragma unroll
-            for (int j = 0; j < NT; ++j)
+                for (int j = 0; j < NT; ++j)
 #pragma unroll
-                for (int e = 0; e < 4; ++e) p[(g4 + 8 * (e >> 1)) * (HD + 2) + j * 8 + 2 * c4 + (e & 1)] = o[j][e];
-            if (c4 == 0)
+                    for (int e = 0; e < 4; ++e) p[(g4 + 8 * (e >> 1)) * (HD + 2) + j * 8 + 2 * c4 + (e & 1)] = o[j][e];
+                if (c4 == 0)
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    p[(g4 + 8 * h) * (HD + 2) + HD] = m_run[h];
-                    p[(g4 + 8 * h) * (HD + 2) + HD + 1] = l_run[h];
+                    for (int h = 0; h < 2; ++h) {
+                        p[(g4 + 8 * h) * (HD + 2) + HD] = m_run[h];
+                        p[(g4 + 8 * h) * (HD + 2) + HD + 1] = l_run[h];
+                    }
+            }
+            rr.consumers_sync(a, lane);
+            if (active && sp == 0) {
+                for (int s = 1; s < n_sp; ++s) {
+                    const float* p = park + (s * n_mt + mt) * PW;
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const int row = g4 + 8 * h;
+                        const float ms = p[row * (HD + 2) + HD], ls = p[row * (HD + 2) + HD + 1];
+                        const float M = fmaxf(m_run[h], ms);
+                        const float Mu = (M == -INFINITY) ? 0.f : M;
+                        const float wa = fast_exp2(m_run[h] - Mu), wb = fast_exp2(ms - Mu);
+#pragma unroll
+                        for (int j = 0; j < NT; ++j) {
+                            o[j][2 * h] = o[j][2 * h] * wa + wb * p[row * (HD + 2) + j * 8 + 2 * c4];
+                            o[j][2 * h + 1] = o[j][2 * h + 1] * wa + wb * p[row * (HD + 2) + j * 8 + 2 * c4 + 1];
+                        }
+                        l_run[h] = l_run[h] * wa + ls * wb;
+                        m_run[h] = M;
+                    }
                 }
-        }
-        __syncthreads();
-        if (!active || sp != 0) return;
-        for (int s = 1; s < n_sp; ++s) {
-            const float* p = park + (s * n_mt + mt) * PW;
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int row = g4 + 8 * h;
-                const float ms = p[row * (HD + 2) + HD], ls = p[row * (HD + 2) + HD + 1];
-                const float M = fmaxf(m_run[h], ms);
-                const float Mu = (M == -INFINITY) ? 0.f : M;
-                const float wa = fast_exp2(m_run[h] - Mu), wb = fast_exp2(ms - Mu);
-#pragma unroll
-                for (int j = 0; j < NT; ++j) {
-                    o[j][2 * h] = o[j][2 * h] * wa + wb * p[row * (HD + 2) + j * 8 + 2 * c4];
-                    o[j][2 * h + 1] = o[j][2 * h + 1] * wa + wb * p[row * (HD + 2) + j * 8 + 2 * c4 + 1];
-                }
-                l_run[h] = l_run[h] * wa + ls * wb;
-                m_run[h] = M;
             }
         }
+        if (!active || sp != 0) return;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-            const int rr = mt * 16 + g4 + 8 * h;
-            if (rr >= u.n_rows) continue;
-            const int item_row = u.row0 + rr;
+            const int r = mt * 16 + g4 + 8 * h;
+            if (r >= u.n_rows) continue;
+            const int item_row = u.row0 + r;
             const int slot = u.slot_base + item_row / a.group;
             const int qh = u.kvh * a.group + item_row % a.group;
             float* dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
@@ -678,53 +728,99 @@ struct TensorPath {
     }
 };
 
+// Producer warp, lane 0: fetch units, publish them, stream their tile pairs.
 template <int HD>
-__global__ void __launch_bounds__(kThreads, 2) decode_kernel(const DecodeArgs a) {
-    extern __shared__ __align__(128) uint8_t ring[];
-    __shared__ __align__(16) Pipe pipe;
-    __shared__ __align__(16) float cc_scratch[4 * kStageTokens * 8];
-    const int tid = threadIdx.x;
-
-    UnitDesc u;
-    {
-        const int* w = a.units + (int64_t)blockIdx.x * kUnitWords;
-        u.tile_off = w[U_TILE_OFF];
-        u.n_tiles = w[U_N_TILES];
-        u.occ_off = w[U_OCC_OFF];
-        u.row0 = w[U_ROW0];
-        u.n_rows = w[U_N_ROWS];
-        u.slot_base = w[U_SLOT_BASE];
-        u.kvh = w[U_KVH];
-        u.kind = w[U_KIND];
+__device__ void produce(const DecodeArgs& a, Ctl& c, uint8_t* ring) {
+    volatile int* abort = &c.abort;
+    int stage = 0;
+    uint32_t phase = 0;
+    for (int k = 0;; ++k) {
+        const int q = k & 1;
+        if (!mbar_wait(smem_u32(&c.uempty[q]), ((k >> 1) & 1) ^ 1)) note_timeout(a, c, 2);
+        int u = *abort ? -1 : a.unit_begin + atomicAdd(a.counter, 1);
+        if (u >= a.unit_end) u = -1;
+        *reinterpret_cast<volatile int*>(&c.unit[q]) = u;
+        mbar_arrive(smem_u32(&c.ufull[q]));
+        if (u < 0) return;
+        const UnitDesc d = load_unit(a, u);
+        const int32_t* tw = a.tiles + d.tile_off;
+        const int n_pairs = (d.n_tiles + 1) / 2;
+        int32_t w[2] = {tw[0], d.n_tiles > 1 ? tw[1] : -1};
+        for (int pr = 0; pr < n_pairs; ++pr) {
+            // next pair's tile words are loaded before this pair's wait
+            const int t2 = 2 * pr + 2;
+            const int32_t nw0 = t2 < d.n_tiles ? tw[t2] : -1, nw1 = t2 + 1 < d.n_tiles ? tw[t2 + 1] : -1;
+            if (!mbar_wait(smem_u32(&c.empty[stage]), phase ^ 1)) note_timeout(a, c, 2);
+            fence_proxy_async();
+            issue_pair<HD>(a, c, d.kvh, ring, w, stage);
+            w[0] = nw0;
+            w[1] = nw1;
+            if (++stage == kStages) {
+                stage = 0;
+                phase ^= 1;
+            }
+        }
     }
+}
+
+template <int HD, int KIND>
+__device__ void consume(const DecodeArgs& a, Ctl& c, uint8_t* ring, float* park, float* scratch) {
+    const int lane = threadIdx.x & 31;
+    RingReader rr{&c, ring, 0, 0, 0};
+    for (int k = 0;; ++k) {
+        const int q = k & 1;
+        if (!mbar_wait(smem_u32(&c.ufull[q]), (k >> 1) & 1)) {
+            note_timeout(a, c, 8);
+            return;
+        }
+        const int u = *reinterpret_cast<volatile int*>(&c.unit[q]);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&c.uempty[q]));
+        if (u < 0) return;
+        const UnitDesc d = load_unit(a, u);
+        if constexpr (KIND == KIND_TENSOR)
+            TensorPath<HD>::unit(a, d, rr, park);
+        else
+            CudaCorePath<HD>::unit(a, d, rr, park, scratch);
+    }
+}
+
+// One persistent launch per unit kind (tensor units come first in the list),
+// so each path gets its own register allocation.
+template <int HD, int KIND>
+__global__ void __launch_bounds__(kDecodeThreads, 2) decode_kernel(const DecodeArgs a) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    __shared__ __align__(16) Ctl ctl;
+    __shared__ __align__(16) float cc_scratch[KIND == KIND_CUDA_CORE ? kConsumerWarps * kStageTokens * 8 : 4];
+    uint8_t* ring = smem;
+    float* park = reinterpret_cast<float*>(smem + Smem<HD>::kRingBytes);
+    const int tid = threadIdx.x, warp = tid >> 5;
     // zero the ring once: rows past a partial block are never copied and must
     // hold finite values (their probabilities are exactly 0)
     {
         uint4* r4 = reinterpret_cast<uint4*>(ring);
-        for (int i = tid; i < Smem<HD>::kBytes / 16; i += kThreads) r4[i] = make_uint4(0, 0, 0, 0);
+        for (int i = tid; i < Smem<HD>::kRingBytes / 16; i += kDecodeThreads) r4[i] = make_uint4(0, 0, 0, 0);
     }
     if (tid == 0) {
-        pipe.abort_at = -1;
-        for (int s = 0; s < kStages; ++s) mbar_init(smem_u32(&pipe.bars[s]), 1);
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(smem_u32(&ctl.full[s]), 1);
+            mbar_init(smem_u32(&ctl.empty[s]), kConsumerWarps);
+        }
+        for (int q = 0; q < 2; ++q) {
+            mbar_init(smem_u32(&ctl.ufull[q]), 1);
+            mbar_init(smem_u32(&ctl.uempty[q]), kConsumerWarps);
+        }
+        mbar_init(smem_u32(&ctl.csync), kConsumerWarps);
+        ctl.abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     fence_proxy_async();
     __syncthreads();
-    if (tid == 0) {
-        const int n_pairs = (u.n_tiles + 1) / 2;
-        int p = 0;
-        for (; p < kStages && p < n_pairs; ++p) issue_pair<HD>(a, u, ring, smem_u32(&pipe.bars[p]), p, p);
-        pipe.issued = p;
+    if (warp == kConsumerWarps) {
+        if ((tid & 31) == 0) produce<HD>(a, ctl, ring);
+        return;
     }
-    if (u.kind == KIND_TENSOR)
-        TensorPath<HD>::run(a, u, ring, &pipe);
-    else
-        CudaCorePath<HD>::run(a, u, ring, &pipe, cc_scratch);
-    // After a wait ran out, let every issued copy land (each wait bounded)
-    // before the CTA exits: pairs abort_at .. issued-1 are outstanding, and
-    // each stage holds at most one of them.
-    if (tid == 0 && pipe.abort_at >= 0)
-        for (int p = pipe.abort_at; p < pipe.issued; ++p) mbar_wait(smem_u32(&pipe.bars[p % kStages]), (p / kStages) & 1);
+    consume<HD, KIND>(a, ctl, ring, park, cc_scratch);
 }
 
 // ------------------------------------------------------------------- merge --
@@ -733,6 +829,7 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
     constexpr int DPL = HD / 32;  // dims per lane: 4 or 2
     const int warp_global = blockIdx.x * 4 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
+    if (blockIdx.x == 0 && threadIdx.x < 2) a.counters[threadIdx.x] = 0;  // decode is done: re-arm its counters
     if (warp_global >= a.n * a.hq) return;
     const int i = warp_global / a.hq, qh = warp_global % a.hq;
     const int beg = a.merge_off[i], end = a.merge_off[i + 1];
@@ -772,11 +869,41 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
     if (lane == 0) a.lse[(int64_t)i * a.hq + qh] = (M + __log2f(L)) * 0.69314718055994531f;
 }
 
+template <int HD, int KIND>
+int decode_grid() {
+    // persistent grid: every resident CTA slot of the device
+    static int grid = [] {
+        int dev = 0, sms = 0, per_sm = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (cudaFuncSetAttribute(decode_kernel<HD, KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 Smem<HD>::kBytes) != cudaSuccess)
+            return 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_kernel<HD, KIND>, kDecodeThreads,
+                                                          Smem<HD>::kBytes) != cudaSuccess)
+            return 0;
+        return sms * std::max(per_sm, 1);
+    }();
+    return grid;
+}
+
+template <int HD, int KIND>
+cudaError_t launch_range(DecodeArgs a, int begin, int end, int32_t* counter, cudaStream_t s) {
+    if (end <= begin) return cudaSuccess;
+    const int slots = decode_grid<HD, KIND>();
+    if (slots == 0) return cudaErrorInvalidConfiguration;
+    a.unit_begin = begin;
+    a.unit_end = end;
+    a.counter = counter;
+    decode_kernel<HD, KIND><<<std::min(end - begin, slots), kDecodeThreads, Smem<HD>::kBytes, s>>>(a);
+    return cudaGetLastError();
+}
+
 template <int HD>
-cudaError_t set_decode_attrs() {
-    static cudaError_t once = cudaFuncSetAttribute(decode_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                   Smem<HD>::kBytes);
-    return once;
+cudaError_t launch_decode_hd(const DecodeArgs& a, cudaStream_t s) {
+    cudaError_t e = launch_range<HD, KIND_TENSOR>(a, 0, a.n_tensor_units, a.counters, s);
+    if (e != cudaSuccess) return e;
+    return launch_range<HD, KIND_CUDA_CORE>(a, a.n_tensor_units, a.n_units, a.counters + 1, s);
 }
 
 }  // namespace
@@ -805,15 +932,7 @@ cudaError_t launch_gather(int hd, const GatherArgs& a, int64_t n_tokens, cudaStr
 
 cudaError_t launch_decode(int hd, const DecodeArgs& a, cudaStream_t s) {
     if (a.n_units == 0) return cudaSuccess;
-    cudaError_t e;
-    if (hd == 64) {
-        if ((e = set_decode_attrs<64>()) != cudaSuccess) return e;
-        decode_kernel<64><<<a.n_units, kThreads, Smem<64>::kBytes, s>>>(a);
-    } else {
-        if ((e = set_decode_attrs<128>()) != cudaSuccess) return e;
-        decode_kernel<128><<<a.n_units, kThreads, Smem<128>::kBytes, s>>>(a);
-    }
-    return cudaGetLastError();
+    return hd == 64 ? launch_decode_hd<64>(a, s) : launch_decode_hd<128>(a, s);
 }
 
 cudaError_t launch_merge(int hd, const MergeArgs& a, cudaStream_t s) {
