@@ -100,7 +100,7 @@ struct Item {
 };
 constexpr int64_t kTargetUnits = 152 * 2 * 6;  // SMs x resident CTAs x waves
 constexpr int32_t kMinChunkTiles = 4;
-constexpr int32_t kMaxChunkTiles = 32;
+constexpr int32_t kMaxChunkTiles = 64;
 }  // namespace
 
 tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t flags, Schedule& S) {

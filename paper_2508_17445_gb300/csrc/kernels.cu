@@ -197,30 +197,19 @@ struct UnitDesc {
     int tile_off, n_tiles, occ_off, row0, n_rows, slot_base, kvh, kind;
 };
 
-__device__ __forceinline__ UnitDesc load_unit(const DecodeArgs& a, int u) {
-    const int* w = a.units + (int64_t)u * kUnitWords;
-    UnitDesc d;
-    d.tile_off = w[U_TILE_OFF];
-    d.n_tiles = w[U_N_TILES];
-    d.occ_off = w[U_OCC_OFF];
-    d.row0 = w[U_ROW0];
-    d.n_rows = w[U_N_ROWS];
-    d.slot_base = w[U_SLOT_BASE];
-    d.kvh = w[U_KVH];
-    d.kind = w[U_KIND];
-    return d;
-}
-
 template <int HD>
 struct Smem {
     static constexpr int kRowBytes = HD * 2;
     static constexpr int kHalfBytes = kStageTokens * kRowBytes;  // K or V of one stage
     static constexpr int kStageBytes = 2 * kHalfBytes;
     static constexpr int kRingBytes = kStages * kStageBytes;
-    // split combine: kConsumerWarps x 16 rows x (HD + 2) floats; the CUDA-core
-    // combine (4 x 8 rows x HD + 64 floats) fits in the same region
-    static constexpr int kParkFloats = kConsumerWarps * 16 * (HD + 2);
-    static constexpr int kBytes = kRingBytes + kParkFloats * 4;
+    // split combine: the (kConsumerWarps - 1) warps that hand over their
+    // state, 16 rows x (HD + 2) floats each; the CUDA-core combine
+    // (4 x 8 rows x HD + 64 floats) fits in the same region
+    static constexpr int kParkFloats = (kConsumerWarps - 1) * 16 * (HD + 2);
+    // the query rows of one tensor unit (64 rows x HD bf16), staged by TMA
+    static constexpr int kQBytes = kConsumerWarps * 16 * HD * 2;
+    static constexpr int kBytes = kRingBytes + kParkFloats * 4 + kQBytes;
 };
 
 // Shared control block of one CTA.
@@ -230,8 +219,11 @@ struct Ctl {
     uint64_t ufull[2];        // unit slot published
     uint64_t uempty[2];       // unit slot read by every consumer warp
     uint64_t csync;           // consumer-only barrier (split combine)
+    uint64_t qfull;           // the current tensor unit's query rows landed
+    uint64_t qempty;          // every consumer warp holds its query fragments
     int valid[kStages][2];    // valid tokens of the stage's two tiles (0: no tile)
-    int unit[2];
+    int unit[2];              // published unit index (-1: no more units)
+    int desc[2][kUnitWords];  // published unit descriptor
     int abort;
 };
 
@@ -280,6 +272,7 @@ struct RingReader {
     int stage;
     uint32_t phase;
     uint32_t sync_phase;
+    uint32_t q_phase;
 
     template <int HD>
     __device__ __forceinline__ const uint8_t* acquire(const DecodeArgs& a, int& v0, int& v1) {
@@ -553,7 +546,8 @@ struct TensorPath {
     static constexpr int KS = HD / 16;  // k-steps of Q.K^T
     static constexpr int NT = HD / 8;   // n-tiles of the output
 
-    __device__ static void unit(const DecodeArgs& a, const UnitDesc& u, RingReader& rr, float* park) {
+    __device__ static void unit(const DecodeArgs& a, const UnitDesc& u, RingReader& rr, float* park,
+                                const uint8_t* qbuf) {
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
         const int n_mt = (u.n_rows + 15) / 16;  // 1..4
         const int n_sp = (n_mt == 1) ? 4 : (n_mt == 2) ? 2 : 1;
@@ -562,28 +556,24 @@ struct TensorPath {
         const int TW = kStageTokens / n_sp;  // 16, 32 or 64 tokens per stage
         const int g4 = lane >> 2, c4 = lane & 3;
 
-        // Q fragments (rows g4 and g4 + 8 of this warp's tile)
+        // Q fragments from the unit's staged query rows (row r of the unit at
+        // qbuf + r * HD * 2); rows past n_rows are zero
         uint32_t qa[KS][4];
-        {
-            const uint16_t* qrow[2] = {nullptr, nullptr};
-            for (int h = 0; h < 2; ++h) {
-                const int r = mt * 16 + g4 + 8 * h;
-                if (active && r < u.n_rows) {
-                    const int item_row = u.row0 + r;
-                    const int occ = a.occ[u.occ_off + item_row / a.group];
-                    const int qh = u.kvh * a.group + item_row % a.group;
-                    qrow[h] = a.q + ((int64_t)occ * a.hq + qh) * HD;
-                }
-            }
+        if (!mbar_wait(smem_u32(&rr.c->qfull), rr.q_phase)) note_timeout(a, *rr.c, 1);
+        rr.q_phase ^= 1;
+        if (active) {
+            const int mi = lane >> 3, ri = lane & 7;
+            const uint32_t qb = smem_u32(qbuf) + (mt * 16 + (mi & 1) * 8 + ri) * (HD * 2) + (mi >> 1) * 16;
+            const bool lo_ok = mt * 16 + g4 < u.n_rows, hi_ok = mt * 16 + g4 + 8 < u.n_rows;
 #pragma unroll
             for (int ks = 0; ks < KS; ++ks) {
-                const int c0 = ks * 16 + 2 * c4;
-                qa[ks][0] = qrow[0] ? *reinterpret_cast<const uint32_t*>(qrow[0] + c0) : 0u;
-                qa[ks][1] = qrow[1] ? *reinterpret_cast<const uint32_t*>(qrow[1] + c0) : 0u;
-                qa[ks][2] = qrow[0] ? *reinterpret_cast<const uint32_t*>(qrow[0] + c0 + 8) : 0u;
-                qa[ks][3] = qrow[1] ? *reinterpret_cast<const uint32_t*>(qrow[1] + c0 + 8) : 0u;
+                ldsm_x4(qb + ks * 32, qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
+                if (!lo_ok) qa[ks][0] = qa[ks][2] = 0u;
+                if (!hi_ok) qa[ks][1] = qa[ks][3] = 0u;
             }
         }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&rr.c->qempty));
         float o[NT][4];
 #pragma unroll
         for (int j = 0; j < NT; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
@@ -676,7 +666,7 @@ struct TensorPath {
             constexpr int PW = 16 * (HD + 2);
             rr.consumers_sync(a, lane);  // the previous unit's combine is done with the park
             if (active && sp > 0) {
-                float* p = park + warp * PW;
+                float* p = park + ((sp - 1) * n_mt + mt) * PW;
 #pragma unroll
                 for (int j = 0; j < NT; ++j)
 #pragma unroll
@@ -691,7 +681,7 @@ struct TensorPath {
             rr.consumers_sync(a, lane);
             if (active && sp == 0) {
                 for (int s = 1; s < n_sp; ++s) {
-                    const float* p = park + (s * n_mt + mt) * PW;
+                    const float* p = park + ((s - 1) * n_mt + mt) * PW;
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
                         const int row = g4 + 8 * h;
@@ -728,45 +718,92 @@ struct TensorPath {
     }
 };
 
-// Producer warp, lane 0: fetch units, publish them, stream their tile pairs.
-template <int HD>
-__device__ void produce(const DecodeArgs& a, Ctl& c, uint8_t* ring) {
+// Producer warp: fetch units, publish them, stage a tensor unit's query rows
+// (one bulk copy per leaf occurrence, lanes in parallel) and stream the
+// unit's tile pairs (lane 0).
+template <int HD, int KIND>
+__device__ void produce(const DecodeArgs& a, Ctl& c, uint8_t* ring, uint8_t* qbuf) {
+    const int lane = threadIdx.x & 31;
     volatile int* abort = &c.abort;
     int stage = 0;
     uint32_t phase = 0;
     for (int k = 0;; ++k) {
         const int q = k & 1;
         if (!mbar_wait(smem_u32(&c.uempty[q]), ((k >> 1) & 1) ^ 1)) note_timeout(a, c, 2);
-        int u = *abort ? -1 : a.unit_begin + atomicAdd(a.counter, 1);
-        if (u >= a.unit_end) u = -1;
-        *reinterpret_cast<volatile int*>(&c.unit[q]) = u;
-        mbar_arrive(smem_u32(&c.ufull[q]));
+        int u = -1;
+        if (lane == 0) {
+            u = *abort ? -1 : a.unit_begin + atomicAdd(a.counter, 1);
+            if (u >= a.unit_end) u = -1;
+        }
+        u = __shfl_sync(0xffffffffu, u, 0);
+        const int word = (u >= 0 && lane < kUnitWords) ? a.units[(int64_t)u * kUnitWords + lane] : 0;
+        UnitDesc d;
+        d.tile_off = __shfl_sync(0xffffffffu, word, U_TILE_OFF);
+        d.n_tiles = __shfl_sync(0xffffffffu, word, U_N_TILES);
+        d.occ_off = __shfl_sync(0xffffffffu, word, U_OCC_OFF);
+        d.row0 = __shfl_sync(0xffffffffu, word, U_ROW0);
+        d.n_rows = __shfl_sync(0xffffffffu, word, U_N_ROWS);
+        d.slot_base = __shfl_sync(0xffffffffu, word, U_SLOT_BASE);
+        d.kvh = __shfl_sync(0xffffffffu, word, U_KVH);
+        d.kind = __shfl_sync(0xffffffffu, word, U_KIND);
+        if (lane == 0) {
+            volatile int* dw = c.desc[q];
+            dw[U_TILE_OFF] = d.tile_off;
+            dw[U_N_TILES] = d.n_tiles;
+            dw[U_OCC_OFF] = d.occ_off;
+            dw[U_ROW0] = d.row0;
+            dw[U_N_ROWS] = d.n_rows;
+            dw[U_SLOT_BASE] = d.slot_base;
+            dw[U_KVH] = d.kvh;
+            dw[U_KIND] = d.kind;
+            *reinterpret_cast<volatile int*>(&c.unit[q]) = u;
+            mbar_arrive(smem_u32(&c.ufull[q]));  // release: descriptor visible to the consumers
+        }
         if (u < 0) return;
-        const UnitDesc d = load_unit(a, u);
-        const int32_t* tw = a.tiles + d.tile_off;
-        const int n_pairs = (d.n_tiles + 1) / 2;
-        int32_t w[2] = {tw[0], d.n_tiles > 1 ? tw[1] : -1};
-        for (int pr = 0; pr < n_pairs; ++pr) {
-            // next pair's tile words are loaded before this pair's wait
-            const int t2 = 2 * pr + 2;
-            const int32_t nw0 = t2 < d.n_tiles ? tw[t2] : -1, nw1 = t2 + 1 < d.n_tiles ? tw[t2 + 1] : -1;
-            if (!mbar_wait(smem_u32(&c.empty[stage]), phase ^ 1)) note_timeout(a, c, 2);
-            fence_proxy_async();
-            issue_pair<HD>(a, c, d.kvh, ring, w, stage);
-            w[0] = nw0;
-            w[1] = nw1;
-            if (++stage == kStages) {
-                stage = 0;
-                phase ^= 1;
+        if constexpr (KIND == KIND_TENSOR) {
+            // query rows of the unit: item rows [row0, row0 + n_rows) of its
+            // occurrence groups, each group's heads contiguous in Q
+            if (!mbar_wait(smem_u32(&c.qempty), (k & 1) ^ 1)) note_timeout(a, c, 2);
+            if (lane == 0) mbar_arrive_expect_tx(smem_u32(&c.qfull), (uint32_t)d.n_rows * HD * 2);
+            __syncwarp();
+            const int g = a.group;
+            const int p_end = (d.row0 + d.n_rows - 1) / g;
+            for (int p = d.row0 / g + lane; p <= p_end; p += 32) {
+                const int r_lo = max(p * g, d.row0), r_hi = min(p * g + g, d.row0 + d.n_rows);
+                const int occ = a.occ[d.occ_off + p];
+                const uint16_t* src = a.q + ((int64_t)occ * a.hq + d.kvh * g + (r_lo - p * g)) * HD;
+                bulk_g2s(smem_u32(qbuf + (r_lo - d.row0) * (HD * 2)), src, (uint32_t)(r_hi - r_lo) * HD * 2,
+                         smem_u32(&c.qfull));
             }
         }
+        if (lane == 0) {
+            const int32_t* tw = a.tiles + d.tile_off;
+            const int n_pairs = (d.n_tiles + 1) / 2;
+            int32_t w[2] = {tw[0], d.n_tiles > 1 ? tw[1] : -1};
+            for (int pr = 0; pr < n_pairs; ++pr) {
+                // next pair's tile words are loaded before this pair's wait
+                const int t2 = 2 * pr + 2;
+                const int32_t nw0 = t2 < d.n_tiles ? tw[t2] : -1, nw1 = t2 + 1 < d.n_tiles ? tw[t2 + 1] : -1;
+                if (!mbar_wait(smem_u32(&c.empty[stage]), phase ^ 1)) note_timeout(a, c, 2);
+                fence_proxy_async();
+                issue_pair<HD>(a, c, d.kvh, ring, w, stage);
+                w[0] = nw0;
+                w[1] = nw1;
+                if (++stage == kStages) {
+                    stage = 0;
+                    phase ^= 1;
+                }
+            }
+        }
+        __syncwarp();
     }
 }
 
 template <int HD, int KIND>
-__device__ void consume(const DecodeArgs& a, Ctl& c, uint8_t* ring, float* park, float* scratch) {
+__device__ void consume(const DecodeArgs& a, Ctl& c, uint8_t* ring, float* park, const uint8_t* qbuf,
+                        float* scratch) {
     const int lane = threadIdx.x & 31;
-    RingReader rr{&c, ring, 0, 0, 0};
+    RingReader rr{&c, ring, 0, 0, 0, 0};
     for (int k = 0;; ++k) {
         const int q = k & 1;
         if (!mbar_wait(smem_u32(&c.ufull[q]), (k >> 1) & 1)) {
@@ -774,12 +811,23 @@ __device__ void consume(const DecodeArgs& a, Ctl& c, uint8_t* ring, float* park,
             return;
         }
         const int u = *reinterpret_cast<volatile int*>(&c.unit[q]);
+        UnitDesc d;
+        {
+            const volatile int* dw = c.desc[q];
+            d.tile_off = dw[U_TILE_OFF];
+            d.n_tiles = dw[U_N_TILES];
+            d.occ_off = dw[U_OCC_OFF];
+            d.row0 = dw[U_ROW0];
+            d.n_rows = dw[U_N_ROWS];
+            d.slot_base = dw[U_SLOT_BASE];
+            d.kvh = dw[U_KVH];
+            d.kind = dw[U_KIND];
+        }
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&c.uempty[q]));
         if (u < 0) return;
-        const UnitDesc d = load_unit(a, u);
         if constexpr (KIND == KIND_TENSOR)
-            TensorPath<HD>::unit(a, d, rr, park);
+            TensorPath<HD>::unit(a, d, rr, park, qbuf);
         else
             CudaCorePath<HD>::unit(a, d, rr, park, scratch);
     }
@@ -794,6 +842,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 2) decode_kernel(const DecodeA
     __shared__ __align__(16) float cc_scratch[KIND == KIND_CUDA_CORE ? kConsumerWarps * kStageTokens * 8 : 4];
     uint8_t* ring = smem;
     float* park = reinterpret_cast<float*>(smem + Smem<HD>::kRingBytes);
+    uint8_t* qbuf = smem + Smem<HD>::kRingBytes + Smem<HD>::kParkFloats * 4;
     const int tid = threadIdx.x, warp = tid >> 5;
     // zero the ring once: rows past a partial block are never copied and must
     // hold finite values (their probabilities are exactly 0)
@@ -811,16 +860,18 @@ __global__ void __launch_bounds__(kDecodeThreads, 2) decode_kernel(const DecodeA
             mbar_init(smem_u32(&ctl.uempty[q]), kConsumerWarps);
         }
         mbar_init(smem_u32(&ctl.csync), kConsumerWarps);
+        mbar_init(smem_u32(&ctl.qfull), 1);
+        mbar_init(smem_u32(&ctl.qempty), kConsumerWarps);
         ctl.abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     fence_proxy_async();
     __syncthreads();
     if (warp == kConsumerWarps) {
-        if ((tid & 31) == 0) produce<HD>(a, ctl, ring);
+        produce<HD, KIND>(a, ctl, ring, qbuf);
         return;
     }
-    consume<HD, KIND>(a, ctl, ring, park, cc_scratch);
+    consume<HD, KIND>(a, ctl, ring, park, qbuf, cc_scratch);
 }
 
 // ------------------------------------------------------------------- merge --
