@@ -203,8 +203,9 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     for (const Item& it : items) {
         if (it.n_tiles == 0) continue;
         const int32_t rows_chunk = (it.n_occ * g * 5 + 3) / 4;
-        const int32_t n_chunks = rows_chunk > chunk ? std::max(1, it.n_tiles / rows_chunk)
-                                                    : (it.n_tiles + chunk - 1) / chunk;
+        const int32_t n_chunks =
+            std::max(rows_chunk > chunk ? std::max(1, it.n_tiles / rows_chunk) : (it.n_tiles + chunk - 1) / chunk,
+                     (it.n_tiles + kMaxUnitTiles - 1) / kMaxUnitTiles);
         const int32_t base = it.n_tiles / n_chunks, extra = it.n_tiles % n_chunks;
         const int32_t rows = it.n_occ * g;
         int32_t toff = it.tile_off;

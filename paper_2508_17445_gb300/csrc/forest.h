@@ -26,6 +26,9 @@ constexpr int32_t kSchedMagic = 0x54505344;
 constexpr int kTensorMinRows = 16;
 // Query rows per tensor-core unit (4 warps x one 16-row MMA tile each).
 constexpr int kTensorRowsPerUnit = 64;
+// Longest unit in pool blocks (the decode kernel keeps a unit's tile words
+// in shared memory).
+constexpr int kMaxUnitTiles = 128;
 // Maximum rows of a CUDA-core unit (two 8-row groups).
 constexpr int kCudaCoreMaxRows = 16;
 // Pool blocks an append kernel launch can address (larger appends loop).

@@ -36,7 +36,9 @@ namespace tp {
 namespace {
 
 constexpr int kConsumerWarps = 4;                          // attention warps per CTA
-constexpr int kDecodeThreads = (kConsumerWarps + 1) * 32;  // + one producer warp
+constexpr int kStreamerWarp = kConsumerWarps;              // issues the K/V bulk copies
+constexpr int kFetcherWarp = kConsumerWarps + 1;           // claims units, stages their data
+constexpr int kDecodeThreads = (kConsumerWarps + 2) * 32;
 constexpr int kBlockTokens = 32;   // tokens per pool block (= tile)
 constexpr int kStageTokens = 64;   // two tiles per pipeline stage
 constexpr int kStages = 2;         // stages in each CTA's shared-memory ring
@@ -183,16 +185,21 @@ __global__ void gather_kernel(const GatherArgs a, int64_t n_tokens) {
 }
 
 // ------------------------------------------------------------------ decode --
-// Persistent, warp-specialised kernel. Each CTA (two per SM) runs one
-// producer warp and kConsumerWarps consumer warps until the global unit
+// Persistent, warp-specialised kernel. Each CTA (two per SM) runs
+// kConsumerWarps consumer warps and two producer warps until the global unit
 // counter runs past the unit list (units are sorted longest first, so the
-// counter hands them out in LPT order). The producer's lane 0 fetches a unit,
-// publishes it in one of two unit slots, and streams the unit's tile pairs
-// into a ring of shared-memory stages with TMA bulk copies; it runs ahead
-// across unit boundaries, so HBM keeps streaming while the consumers finish a
-// unit (the split combine and partial stores). Every wait is an mbarrier wait
-// bounded in time; a wait that runs out sets the device error flag and the
-// kernel carries on to a bounded exit.
+// counter hands them out in LPT order):
+//   fetcher   claims the next unit, publishes its descriptor and tile words
+//             in one of two shared-memory unit slots and stages a tensor
+//             unit's query rows with TMA -- up to two units ahead;
+//   streamer  (one lane) streams the published units' tile pairs into a ring
+//             of shared-memory stages with TMA bulk copies, with nothing but
+//             stage waits between one unit and the next, so HBM keeps
+//             streaming while the consumers finish a unit (split combine,
+//             partial stores);
+//   consumers run the attention math on each stage.
+// Every wait is an mbarrier wait bounded in time; a wait that runs out sets
+// the device error flag and the kernel carries on to a bounded exit.
 struct UnitDesc {
     int tile_off, n_tiles, occ_off, row0, n_rows, slot_base, kvh, kind;
 };
@@ -224,6 +231,7 @@ struct Ctl {
     int valid[kStages][2];    // valid tokens of the stage's two tiles (0: no tile)
     int unit[2];              // published unit index (-1: no more units)
     int desc[2][kUnitWords];  // published unit descriptor
+    int tiles[2][kMaxUnitTiles];  // published unit's tile words
     int abort;
 };
 
@@ -718,17 +726,16 @@ struct TensorPath {
     }
 };
 
-// Producer warp: fetch units, publish them, stage a tensor unit's query rows
-// (one bulk copy per leaf occurrence, lanes in parallel) and stream the
-// unit's tile pairs (lane 0).
+// Fetcher warp: claim units, publish descriptor + tile words, stage a tensor
+// unit's query rows (one bulk copy per leaf occurrence group, lanes in
+// parallel).
 template <int HD, int KIND>
-__device__ void produce(const DecodeArgs& a, Ctl& c, uint8_t* ring, uint8_t* qbuf) {
+__device__ void fetch_units(const DecodeArgs& a, Ctl& c, uint8_t* qbuf) {
     const int lane = threadIdx.x & 31;
     volatile int* abort = &c.abort;
-    int stage = 0;
-    uint32_t phase = 0;
     for (int k = 0;; ++k) {
         const int q = k & 1;
+        // the slot is free once the consumers and the streamer are done with unit k-2
         if (!mbar_wait(smem_u32(&c.uempty[q]), ((k >> 1) & 1) ^ 1)) note_timeout(a, c, 2);
         int u = -1;
         if (lane == 0) {
@@ -746,6 +753,8 @@ __device__ void produce(const DecodeArgs& a, Ctl& c, uint8_t* ring, uint8_t* qbu
         d.slot_base = __shfl_sync(0xffffffffu, word, U_SLOT_BASE);
         d.kvh = __shfl_sync(0xffffffffu, word, U_KVH);
         d.kind = __shfl_sync(0xffffffffu, word, U_KIND);
+        if (u >= 0)
+            for (int t = lane; t < d.n_tiles; t += 32) c.tiles[q][t] = a.tiles[d.tile_off + t];
         if (lane == 0) {
             volatile int* dw = c.desc[q];
             dw[U_TILE_OFF] = d.tile_off;
@@ -757,8 +766,10 @@ __device__ void produce(const DecodeArgs& a, Ctl& c, uint8_t* ring, uint8_t* qbu
             dw[U_KVH] = d.kvh;
             dw[U_KIND] = d.kind;
             *reinterpret_cast<volatile int*>(&c.unit[q]) = u;
-            mbar_arrive(smem_u32(&c.ufull[q]));  // release: descriptor visible to the consumers
         }
+        __threadfence_block();  // every lane's tile-word stores, before lane 0 publishes
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&c.ufull[q]));  // release: slot visible to its readers
         if (u < 0) return;
         if constexpr (KIND == KIND_TENSOR) {
             // query rows of the unit: item rows [row0, row0 + n_rows) of its
@@ -776,26 +787,37 @@ __device__ void produce(const DecodeArgs& a, Ctl& c, uint8_t* ring, uint8_t* qbu
                          smem_u32(&c.qfull));
             }
         }
-        if (lane == 0) {
-            const int32_t* tw = a.tiles + d.tile_off;
-            const int n_pairs = (d.n_tiles + 1) / 2;
-            int32_t w[2] = {tw[0], d.n_tiles > 1 ? tw[1] : -1};
-            for (int pr = 0; pr < n_pairs; ++pr) {
-                // next pair's tile words are loaded before this pair's wait
-                const int t2 = 2 * pr + 2;
-                const int32_t nw0 = t2 < d.n_tiles ? tw[t2] : -1, nw1 = t2 + 1 < d.n_tiles ? tw[t2 + 1] : -1;
-                if (!mbar_wait(smem_u32(&c.empty[stage]), phase ^ 1)) note_timeout(a, c, 2);
-                fence_proxy_async();
-                issue_pair<HD>(a, c, d.kvh, ring, w, stage);
-                w[0] = nw0;
-                w[1] = nw1;
-                if (++stage == kStages) {
-                    stage = 0;
-                    phase ^= 1;
-                }
+    }
+}
+
+// Streamer (one lane): stream the tile pairs of each published unit.
+template <int HD>
+__device__ void stream_units(const DecodeArgs& a, Ctl& c, uint8_t* ring) {
+    int stage = 0;
+    uint32_t phase = 0;
+    for (int k = 0;; ++k) {
+        const int q = k & 1;
+        if (!mbar_wait(smem_u32(&c.ufull[q]), (k >> 1) & 1)) {
+            note_timeout(a, c, 2);
+            return;
+        }
+        const int u = *reinterpret_cast<volatile int*>(&c.unit[q]);
+        if (u < 0) return;
+        const int n_tiles = *reinterpret_cast<volatile int*>(&c.desc[q][U_N_TILES]);
+        const int kvh = *reinterpret_cast<volatile int*>(&c.desc[q][U_KVH]);
+        const volatile int* tw = c.tiles[q];
+        const int n_pairs = (n_tiles + 1) / 2;
+        for (int pr = 0; pr < n_pairs; ++pr) {
+            const int32_t w[2] = {tw[2 * pr], 2 * pr + 1 < n_tiles ? tw[2 * pr + 1] : -1};
+            if (!mbar_wait(smem_u32(&c.empty[stage]), phase ^ 1)) note_timeout(a, c, 2);
+            fence_proxy_async();
+            issue_pair<HD>(a, c, kvh, ring, w, stage);
+            if (++stage == kStages) {
+                stage = 0;
+                phase ^= 1;
             }
         }
-        __syncwarp();
+        mbar_arrive(smem_u32(&c.uempty[q]));  // done with the slot's tile words
     }
 }
 
@@ -857,7 +879,7 @@ __global__ void __launch_bounds__(kDecodeThreads, 2) decode_kernel(const DecodeA
         }
         for (int q = 0; q < 2; ++q) {
             mbar_init(smem_u32(&ctl.ufull[q]), 1);
-            mbar_init(smem_u32(&ctl.uempty[q]), kConsumerWarps);
+            mbar_init(smem_u32(&ctl.uempty[q]), kConsumerWarps + 1);  // consumers + streamer
         }
         mbar_init(smem_u32(&ctl.csync), kConsumerWarps);
         mbar_init(smem_u32(&ctl.qfull), 1);
@@ -867,8 +889,12 @@ __global__ void __launch_bounds__(kDecodeThreads, 2) decode_kernel(const DecodeA
     }
     fence_proxy_async();
     __syncthreads();
-    if (warp == kConsumerWarps) {
-        produce<HD, KIND>(a, ctl, ring, qbuf);
+    if (warp == kStreamerWarp) {
+        if ((tid & 31) == 0) stream_units<HD>(a, ctl, ring);
+        return;
+    }
+    if (warp == kFetcherWarp) {
+        fetch_units<HD, KIND>(a, ctl, qbuf);
         return;
     }
     consume<HD, KIND>(a, ctl, ring, park, qbuf, cc_scratch);
