@@ -158,6 +158,34 @@ tp_status tp_decode(tp_tree* tree, const tp_node* leaves, int32_t n, const void*
 tp_status tp_decode_ex(tp_tree* tree, const tp_node* leaves, int32_t n, const void* Q, void* O,
                        float* LSE, uint32_t flags);
 
+/*
+ * tp_decode_ex without any device allocation. The paper has no counterpart:
+ * this entry point exists for callers that cannot call cudaMalloc on the
+ * decode path -- e.g. a serving process whose device memory is carved up at
+ * start-up (the KV pool, weights, activations) and that forbids later
+ * allocations, or a latency-critical loop that cannot afford cudaMalloc's
+ * implicit device synchronisation. tp_decode_ex keeps its schedule and
+ * partial results in buffers it grows with cudaMalloc; this variant keeps
+ * them in one statically sized device array of TP_NOALLOC_SCRATCH_BYTES that
+ * the library declares at file scope (every GPU that loads the library holds
+ * it until the process exits) and calls no cudaMalloc, cudaFree or other
+ * allocating routine. Arguments and results are those of tp_decode_ex.
+ *   - A call whose schedule plus fp32 partials need more than
+ *     TP_NOALLOC_SCRATCH_BYTES returns TP_ERR_OOM and launches nothing.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current); make that first
+ *     call before any stream capture.
+ *   - Every call in the process shares the one array and it keeps the last
+ *     call's contents; the unit counters that must start at zero are
+ *     cleared by each call. Calls whose device work overlaps -- on two
+ *     streams, or from two trees -- race on the array and must not overlap.
+ *   - The schedule is copied from pageable host memory, so the call waits
+ *     for the tree's stream to drain that far before it returns.
+ */
+#define TP_NOALLOC_SCRATCH_BYTES (32ll << 20)
+tp_status tp_decode_noalloc(tp_tree* tree, const tp_node* leaves, int32_t n, const void* Q, void* O,
+                            float* LSE, uint32_t flags);
+
 /* Wait for the tree's stream; TP_ERR_DEVICE if a kernel gave up a bounded
  * wait since the last tp_sync (the flag is then cleared), TP_ERR_CUDA on a
  * CUDA error. */

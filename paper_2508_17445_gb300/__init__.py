@@ -23,7 +23,7 @@ __all__ = [
     "tp_set_stream", "tp_add_root", "tp_append_segment", "tp_fork", "tp_prune", "tp_decode", "tp_decode_ex",
     "tp_sync", "tp_last_error", "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop",
     "tp_debug_path", "tp_debug_gather",
-    "tp_debug_schedule", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE",
+    "tp_debug_schedule", "tp_decode_noalloc", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE",
     "EXPORTED_SYMBOLS",
 ]
 
@@ -42,7 +42,7 @@ EXPORTED_SYMBOLS = (
     "tp_pool_bytes", "tp_tree_create", "tp_tree_destroy", "tp_set_stream", "tp_add_root",
     "tp_append_segment", "tp_fork", "tp_prune", "tp_decode", "tp_decode_ex", "tp_sync", "tp_last_error",
     "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop", "tp_debug_path",
-    "tp_debug_gather", "tp_debug_schedule",
+    "tp_debug_gather", "tp_debug_schedule", "tp_decode_noalloc",
 )
 
 
@@ -101,6 +101,7 @@ def load_library() -> ctypes.CDLL:
         "tp_prune": (I32, [P, I32]),
         "tp_decode": (I32, [P, P, I32, P, P, P]),
         "tp_decode_ex": (I32, [P, P, I32, P, P, P, U32]),
+        "tp_decode_noalloc": (I32, [P, P, I32, P, P, P, U32]),
         "tp_sync": (I32, [P]),
         "tp_last_error": (ctypes.c_char_p, [P]),
         "tp_get_node_info": (I32, [P, I32, P]),
@@ -183,6 +184,12 @@ def tp_decode_ex(h, leaves: Sequence[int], Q, O, LSE, flags: int = 0) -> None:
 def tp_decode(h, leaves: Sequence[int], Q, O, LSE) -> None:
     arr = _node_array(leaves)
     _check(h, load_library().tp_decode(h, arr.ctypes.data, len(arr), _ptr(Q), _ptr(O), _ptr(LSE)))
+
+
+def tp_decode_noalloc(h, leaves: Sequence[int], Q, O, LSE, flags: int = 0) -> None:
+    """tp_decode_ex without device allocation (scratch in the library's static array)."""
+    arr = _node_array(leaves)
+    _check(h, load_library().tp_decode_noalloc(h, arr.ctypes.data, len(arr), _ptr(Q), _ptr(O), _ptr(LSE), flags))
 
 
 def tp_sync(h) -> None:

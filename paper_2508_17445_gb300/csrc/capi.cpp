@@ -352,6 +352,73 @@ tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void*
     return TP_OK;
 }
 
+tp_status tp_decode_noalloc(tp_tree* t, const tp_node* leaves, int32_t n, const void* Q, void* O, float* LSE,
+                            uint32_t flags) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    if (n < 0) return fail(t, TP_ERR_INVALID_ARG, "n < 0");
+    if (n == 0) return TP_OK;
+    if (!leaves) return fail(t, TP_ERR_INVALID_ARG, "leaves is NULL");
+    if (!t->cfg.pool) return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree cannot decode");
+    if (!Q || !O || !LSE || !aligned(Q, 16) || !aligned(O, 16) || !aligned(LSE, 4))
+        return fail(t, TP_ERR_INVALID_ARG, "Q/O must be 16-byte and LSE 4-byte aligned device pointers");
+    tp::Schedule S;  // host-side only; the tree's schedule cache is left alone
+    tp_status st = tp::build_schedule(t, leaves, n, flags & ~TP_DECODE_NO_CACHE, S);
+    if (st != TP_OK) return st;
+    const int32_t hq = t->cfg.num_q_heads, hd = t->cfg.head_dim;
+    const int64_t sched_bytes = ((int64_t)S.words.size() * 4 + 255) / 256 * 256;
+    const int64_t part_bytes = (int64_t)S.n_slots * hq * (hd + 1) * 4;
+    if (sched_bytes + part_bytes > TP_NOALLOC_SCRATCH_BYTES)
+        return fail(t, TP_ERR_OOM,
+                    "tp_decode_noalloc needs " + std::to_string(sched_bytes + part_bytes) +
+                        " bytes of static scratch; the library holds " + std::to_string(TP_NOALLOC_SCRATCH_BYTES) +
+                        " (decode fewer leaves per call, or use tp_decode_ex)");
+    void* base = nullptr;
+    cudaError_t e = tp::noalloc_scratch(&base);
+    if (e != cudaSuccess) return cuda_fail(t, e, "static scratch address");
+    int32_t* d_sched = (int32_t*)base;
+    float* d_part = (float*)((uint8_t*)base + sched_bytes);
+    e = cudaMemcpyAsync(d_sched, S.words.data(), S.words.size() * 4, cudaMemcpyHostToDevice, t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "schedule upload");
+    e = cudaMemsetAsync(t->d_err + 1, 0, 2 * sizeof(int32_t), t->stream);  // unit counters start at zero
+    if (e != cudaSuccess) return cuda_fail(t, e, "counter reset");
+
+    tp::DecodeArgs a;
+    a.units = d_sched + S.off_units;
+    a.tiles = d_sched + S.off_tiles;
+    a.occ = d_sched + S.off_occ;
+    a.q = (const uint16_t*)Q;
+    a.pool = (const uint8_t*)t->cfg.pool;
+    a.part_o = d_part;
+    a.part_lse = d_part + (int64_t)S.n_slots * hq * hd;
+    a.err = t->d_err;
+    a.counters = t->d_err + 1;
+    a.counter = nullptr;
+    a.n_tensor_units = S.n_tensor;
+    a.unit_begin = a.unit_end = 0;
+    a.head_bytes = t->cfg.block_tokens * hd * 2;
+    a.block_bytes = (int64_t)2 * t->cfg.num_kv_heads * a.head_bytes;
+    a.n_units = S.n_units;
+    a.hq = hq;
+    a.hkv = t->cfg.num_kv_heads;
+    a.group = hq / t->cfg.num_kv_heads;
+    a.qk_scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
+    e = tp::launch_decode(hd, a, t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "decode kernel");
+    tp::MergeArgs m;
+    m.merge_off = d_sched + S.off_merge_off;
+    m.merge_slot = d_sched + S.off_merge_slot;
+    m.part_o = a.part_o;
+    m.part_lse = a.part_lse;
+    m.out = (uint16_t*)O;
+    m.lse = LSE;
+    m.counters = t->d_err + 1;
+    m.n = n;
+    m.hq = hq;
+    e = tp::launch_merge(hd, m, t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "merge kernel");
+    return TP_OK;
+}
+
 tp_status tp_decode(tp_tree* t, const tp_node* leaves, int32_t n, const void* Q, void* O, float* LSE) {
     return tp_decode_ex(t, leaves, n, Q, O, LSE, 0u);
 }

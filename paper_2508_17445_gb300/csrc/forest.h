@@ -99,6 +99,8 @@ cudaError_t launch_decode(int head_dim, const DecodeArgs& a, cudaStream_t s);
 cudaError_t launch_merge(int head_dim, const MergeArgs& a, cudaStream_t s);
 cudaError_t launch_gather(int head_dim, const GatherArgs& a, int64_t n_tokens, cudaStream_t s);
 int decode_smem_bytes(int head_dim);
+// Device address of the library's static scratch array (tp_decode_noalloc).
+cudaError_t noalloc_scratch(void** device_ptr);
 
 // ---- host objects ---------------------------------------------------------
 struct Node {

@@ -29,6 +29,7 @@
 #include <stdint.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "forest.h"
 
@@ -986,6 +987,33 @@ cudaError_t launch_decode_hd(const DecodeArgs& a, cudaStream_t s) {
 }  // namespace
 
 int decode_smem_bytes(int head_dim) { return head_dim == 64 ? Smem<64>::kBytes : Smem<128>::kBytes; }
+
+// ------------------------------------------------------- static scratch --
+// Scratch of tp_decode_noalloc (schedule words, then fp32 partials): a
+// file-scope device array, so that entry point never allocates. Device code
+// could name it directly; host code only sees a host-side stand-in for it,
+// so the launchers take the device address that cudaGetSymbolAddress gives,
+// looked up once per device with that device current.
+static __device__ __align__(256) uint8_t g_noalloc_scratch[TP_NOALLOC_SCRATCH_BYTES];
+
+cudaError_t noalloc_scratch(void** device_ptr) {
+    constexpr int kMaxDevices = 64;
+    static void* addr[kMaxDevices] = {};
+    static std::mutex lock;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> g(lock);
+    if (!addr[dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess) return e;
+        addr[dev] = p;
+    }
+    *device_ptr = addr[dev];
+    return cudaSuccess;
+}
 
 cudaError_t launch_append(int hd, const AppendArgs& a, cudaStream_t s) {
     const int64_t chunks = 2ll * a.n_tokens * a.hkv * (hd / 8);
