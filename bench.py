@@ -91,6 +91,27 @@ def make_script(args, seed):
     return workloads.by_name(args.workload, **kw)
 
 
+def shard_seed(seed, rank):
+    """Rank r of a multi-GPU job decodes its own forest: prompts drawn with
+    seed + r, so ranks hold independent trees and share nothing."""
+    return seed + rank
+
+
+def max_over_ranks(values, device="cpu"):
+    """Element-wise max over ranks (the job's time is its slowest rank's)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor(values, dtype=torch.float64, device=device)
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def job_rate(leaves_per_rank, world, steps, ms_total):
+    """Whole-job leaf-queries/s: every rank's leaves, over the slowest rank's time."""
+    return leaves_per_rank * world * steps / (ms_total / 1e3)
+
+
 def workload_label(script):
     h = script.heads
     return f"{script.name}: {script.description}; {h.num_q_heads} q / {h.num_kv_heads} kv heads, head_dim {h.head_dim}, bf16"
@@ -188,72 +209,84 @@ class ClockSampler:
 # --------------------------------------------------------------------------
 # CPU oracle timing (the reported baseline; never on the product path)
 # --------------------------------------------------------------------------
-def oracle_rate(script, kv_device, budget_s, rng_seed=0):
-    """Leaf-queries/s of the fp64 oracle on a bounded sample of leaves, all
-    host cores. K/V of the sampled paths are fetched before timing."""
-    import numpy as np
-    import torch
+class OracleTimer:
+    """Times the fp64 oracle on leaf samples of one forest, on all host cores.
+    K/V of sampled paths are fetched into a host cache before timing."""
 
-    import oracle
+    def __init__(self, script, kv_device):
+        import oracle
+        self.oracle = oracle
+        self.script = script
+        self.kv_device = kv_device
+        self.model = oracle.OracleForest(block_tokens=32, pool_blocks=script.upper_bound_blocks(32) + 64).replay(script)
+        self.q = script.q("cpu")
+        self.cores = os.cpu_count() or 1
+        self.cache = {}
 
-    model = oracle.OracleForest(block_tokens=32, pool_blocks=script.upper_bound_blocks(32) + 64).replay(script)
-    n = len(script.leaves)
-    rng = np.random.default_rng(rng_seed)
-    order = rng.permutation(n).tolist()
-    q = script.q("cpu")
-    cores = os.cpu_count() or 1
-    cache = {}
-
-    def fetch(rows):
+    def fetch(self, rows):
         for i in rows:
-            for kv_id in model.path_chunks(script.leaves[i]):
-                if kv_id not in cache:
-                    k, v = script.kv(kv_id, kv_device)
-                    cache[kv_id] = (oracle.bf16_bits(k.cpu()), oracle.bf16_bits(v.cpu()))
+            for kv_id in self.model.path_chunks(self.script.leaves[i]):
+                if kv_id not in self.cache:
+                    k, v = self.script.kv(kv_id, self.kv_device)
+                    self.cache[kv_id] = (self.oracle.bf16_bits(k.cpu()), self.oracle.bf16_bits(v.cpu()))
 
-    def run(rows):
+    def seconds(self, rows):
+        self.fetch(rows)
         t0 = time.perf_counter()
-        model.decode(script.leaves, q, lambda i: cache[i], threads=cores, indices=rows)
+        self.model.decode(self.script.leaves, self.q, lambda i: self.cache[i], threads=self.cores, indices=rows)
         return time.perf_counter() - t0
 
-    probe = order[: min(n, max(cores, 8))]
-    fetch(probe)
-    dt = run(probe)
-    per_leaf = dt / len(probe)
-    k = int(min(n, max(len(probe), budget_s / max(per_leaf, 1e-9))))
-    rows = order[:k]
-    fetch(rows)
-    dt = run(rows)
-    return {"value": k / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"{k} of {n} leaves of the same forest, fp64 C oracle (path materialised, naive "
-                      f"softmax attention), threads over leaves; {dt:.1f} s", "seconds": dt, "leaves": k}
+    def sample(self, budget_s, rng_seed):
+        """A seeded leaf sample sized to about budget_s of oracle work."""
+        import numpy as np
+        n = len(self.script.leaves)
+        order = np.random.default_rng(rng_seed).permutation(n).tolist()
+        if not hasattr(self, "per_leaf"):
+            probe = order[: min(n, max(self.cores, 8))]
+            self.per_leaf = self.seconds(probe) / len(probe)
+        k = int(min(n, max(min(n, self.cores), budget_s / max(self.per_leaf, 1e-9))))
+        return order[:k]
+
+
+def oracle_rate(script, kv_device, budget_s, rng_seed=0):
+    """Leaf-queries/s of the fp64 oracle on a bounded sample of leaves."""
+    t = OracleTimer(script, kv_device)
+    rows = t.sample(budget_s, rng_seed)
+    dt = t.seconds(rows)
+    n = len(script.leaves)
+    return {"value": len(rows) / dt, "unit": UNIT, "cores": t.cores, "kind": "oracle",
+            "sample": f"{len(rows)} of {n} leaves of the same forest, fp64 C oracle (path materialised, naive "
+                      f"softmax attention), threads over leaves; {dt:.1f} s", "seconds": dt, "leaves": len(rows)}
 
 
 def run_reference(args, rank, world):
-    """--impl reference: the CPU oracle on the host cores, same metric/config."""
+    """--impl reference: the CPU oracle on the host cores, same metric/config.
+    Each step decodes a seeded leaf sample sized so warm-up + steps take a
+    few minutes; the rate is sampled leaves / oracle time."""
     if rank != 0:
         return
     script = make_script(args, args.seed)
     desc = describe(script)
-    # each step: a bounded sample sized so warmup + steps take a few minutes
     per_step_budget = max(1.0, 150.0 / max(1, args.steps + args.warmup))
-    probe = oracle_rate(script, "cpu", per_step_budget, rng_seed=0)
-    k = probe["leaves"]
-    times = []
+    timer = OracleTimer(script, "cpu")
+    leaves_done, secs, ks = 0, 0.0, []
     for step in range(args.warmup + args.steps):
-        r = oracle_rate(script, "cpu", per_step_budget, rng_seed=step + 1)
+        rows = timer.sample(per_step_budget, rng_seed=step)
+        dt = timer.seconds(rows)
         if step >= args.warmup:
-            times.append(r["seconds"] / r["leaves"])
-    per_leaf = sum(times) / len(times)
-    value = 1.0 / per_leaf
+            leaves_done += len(rows)
+            secs += dt
+            ks.append(len(rows))
+    value = leaves_done / secs
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_leaf * desc["leaves"] * 1e3,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": desc["leaves"] / value * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": workload_label(script), "leaves": desc["leaves"],
                    "unique_kv_bytes": desc["unique_kv_bytes"]},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": probe["cores"], "kind": "oracle",
-                         "sample": f"each step: about {k} of {desc['leaves']} leaves, fp64 C oracle on host cores"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": timer.cores, "kind": "oracle",
+                         "sample": f"each step: {min(ks)}-{max(ks)} of {desc['leaves']} leaves (seeded sample), "
+                                   f"fp64 C oracle, threads over leaves; ms_per_step scaled to all leaves"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -287,7 +320,7 @@ def main():
     if world > 1:
         dist.barrier()
 
-    script = make_script(args, args.seed + rank)
+    script = make_script(args, shard_seed(args.seed, rank))
     desc = describe(script)
     h = script.heads
     t_setup = time.perf_counter()
@@ -363,15 +396,12 @@ def main():
     forest.sync()
 
     # ---- max over ranks
-    vals = torch.tensor([ms_total, ms_uncached, ms_noshare, e2e_s], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(vals, op=dist.ReduceOp.MAX)
-    ms_total, ms_uncached, ms_noshare, e2e_s = vals.tolist()
+    ms_total, ms_uncached, ms_noshare, e2e_s = max_over_ranks([ms_total, ms_uncached, ms_noshare, e2e_s], dev)
     leaves_all = n * world
 
     if rank == 0:
         ms_step = ms_total / args.steps
-        value = leaves_all * args.steps / (ms_total / 1e3)
+        value = job_rate(n, world, args.steps, ms_total)
         peak, peak_kind = peaks()
         dec = ktimes["decode"]
         mer = ktimes["merge"]
