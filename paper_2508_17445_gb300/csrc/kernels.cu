@@ -212,11 +212,17 @@ struct Smem {
     static constexpr int kStageBytes = 2 * kHalfBytes;
     static constexpr int kRingBytes = kStages * kStageBytes;
     // split combine: the (kConsumerWarps - 1) warps that hand over their
-    // state, 16 rows x (HD + 2) floats each; the CUDA-core combine
-    // (4 x 8 rows x HD + 64 floats) fits in the same region
-    static constexpr int kParkFloats = (kConsumerWarps - 1) * 16 * (HD + 2);
-    // the query rows of one tensor unit (64 rows x HD bf16), staged by TMA
-    static constexpr int kQBytes = kConsumerWarps * 16 * HD * 2;
+    // state, 16 rows x kParkPitch floats each (o in columns [0, HD), m and l
+    // in HD and HD + 1; the pitch makes the float2 accesses of a half warp
+    // hit 32 distinct banks); the CUDA-core combine (4 x 8 rows x HD + 64
+    // floats) fits in the same region
+    static constexpr int kParkPitch = HD + 8;
+    static constexpr int kParkFloats = (kConsumerWarps - 1) * 16 * kParkPitch;
+    // the query rows of one tensor unit (64 rows x HD bf16), staged by TMA one
+    // row per copy at a 16-byte-padded pitch so ldmatrix rows fall in
+    // distinct bank groups
+    static constexpr int kQPitch = HD * 2 + 16;
+    static constexpr int kQBytes = kConsumerWarps * 16 * kQPitch;
     static constexpr int kBytes = kRingBytes + kParkFloats * 4 + kQBytes;
 };
 
@@ -572,7 +578,7 @@ struct TensorPath {
         rr.q_phase ^= 1;
         if (active) {
             const int mi = lane >> 3, ri = lane & 7;
-            const uint32_t qb = smem_u32(qbuf) + (mt * 16 + (mi & 1) * 8 + ri) * (HD * 2) + (mi >> 1) * 16;
+            const uint32_t qb = smem_u32(qbuf) + (mt * 16 + (mi & 1) * 8 + ri) * Smem<HD>::kQPitch + (mi >> 1) * 16;
             const bool lo_ok = mt * 16 + g4 < u.n_rows, hi_ok = mt * 16 + g4 + 8 < u.n_rows;
 #pragma unroll
             for (int ks = 0; ks < KS; ++ks) {
@@ -671,21 +677,22 @@ struct TensorPath {
             l_run[h] += __shfl_xor_sync(0xffffffffu, l_run[h], 2);
         }
         if (n_sp > 1) {
-            // token splits of one M-tile meet in shared memory: [warp][16 rows][HD + 2]
-            constexpr int PW = 16 * (HD + 2);
+            // token splits of one M-tile meet in shared memory: [warp][16 rows][pitch]
+            constexpr int PP = Smem<HD>::kParkPitch;
+            constexpr int PW = 16 * PP;
             rr.consumers_sync(a, lane);  // the previous unit's combine is done with the park
             if (active && sp > 0) {
                 float* p = park + ((sp - 1) * n_mt + mt) * PW;
 #pragma unroll
                 for (int j = 0; j < NT; ++j)
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) p[(g4 + 8 * (e >> 1)) * (HD + 2) + j * 8 + 2 * c4 + (e & 1)] = o[j][e];
+                    for (int h = 0; h < 2; ++h)
+                        *reinterpret_cast<float2*>(&p[(g4 + 8 * h) * PP + j * 8 + 2 * c4]) =
+                            make_float2(o[j][2 * h], o[j][2 * h + 1]);
                 if (c4 == 0)
 #pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        p[(g4 + 8 * h) * (HD + 2) + HD] = m_run[h];
-                        p[(g4 + 8 * h) * (HD + 2) + HD + 1] = l_run[h];
-                    }
+                    for (int h = 0; h < 2; ++h)
+                        *reinterpret_cast<float2*>(&p[(g4 + 8 * h) * PP + HD]) = make_float2(m_run[h], l_run[h]);
             }
             rr.consumers_sync(a, lane);
             if (active && sp == 0) {
@@ -694,14 +701,16 @@ struct TensorPath {
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
                         const int row = g4 + 8 * h;
-                        const float ms = p[row * (HD + 2) + HD], ls = p[row * (HD + 2) + HD + 1];
+                        const float2 ml = *reinterpret_cast<const float2*>(&p[row * PP + HD]);
+                        const float ms = ml.x, ls = ml.y;
                         const float M = fmaxf(m_run[h], ms);
                         const float Mu = (M == -INFINITY) ? 0.f : M;
                         const float wa = fast_exp2(m_run[h] - Mu), wb = fast_exp2(ms - Mu);
 #pragma unroll
                         for (int j = 0; j < NT; ++j) {
-                            o[j][2 * h] = o[j][2 * h] * wa + wb * p[row * (HD + 2) + j * 8 + 2 * c4];
-                            o[j][2 * h + 1] = o[j][2 * h + 1] * wa + wb * p[row * (HD + 2) + j * 8 + 2 * c4 + 1];
+                            const float2 x = *reinterpret_cast<const float2*>(&p[row * PP + j * 8 + 2 * c4]);
+                            o[j][2 * h] = o[j][2 * h] * wa + wb * x.x;
+                            o[j][2 * h + 1] = o[j][2 * h + 1] * wa + wb * x.y;
                         }
                         l_run[h] = l_run[h] * wa + ls * wb;
                         m_run[h] = M;
@@ -773,19 +782,17 @@ __device__ void fetch_units(const DecodeArgs& a, Ctl& c, uint8_t* qbuf) {
         if (lane == 0) mbar_arrive(smem_u32(&c.ufull[q]));  // release: slot visible to its readers
         if (u < 0) return;
         if constexpr (KIND == KIND_TENSOR) {
-            // query rows of the unit: item rows [row0, row0 + n_rows) of its
-            // occurrence groups, each group's heads contiguous in Q
+            // query rows of the unit: item row row0 + r is q-head
+            // kvh * g + (row0 + r) % g of occurrence occ[(row0 + r) / g]
             if (!mbar_wait(smem_u32(&c.qempty), (k & 1) ^ 1)) note_timeout(a, c, 2);
             if (lane == 0) mbar_arrive_expect_tx(smem_u32(&c.qfull), (uint32_t)d.n_rows * HD * 2);
             __syncwarp();
             const int g = a.group;
-            const int p_end = (d.row0 + d.n_rows - 1) / g;
-            for (int p = d.row0 / g + lane; p <= p_end; p += 32) {
-                const int r_lo = max(p * g, d.row0), r_hi = min(p * g + g, d.row0 + d.n_rows);
-                const int occ = a.occ[d.occ_off + p];
-                const uint16_t* src = a.q + ((int64_t)occ * a.hq + d.kvh * g + (r_lo - p * g)) * HD;
-                bulk_g2s(smem_u32(qbuf + (r_lo - d.row0) * (HD * 2)), src, (uint32_t)(r_hi - r_lo) * HD * 2,
-                         smem_u32(&c.qfull));
+            for (int r = lane; r < d.n_rows; r += 32) {  // one 2*HD-byte copy per row
+                const int item_row = d.row0 + r;
+                const int occ = a.occ[d.occ_off + item_row / g];
+                const uint16_t* src = a.q + ((int64_t)occ * a.hq + d.kvh * g + item_row % g) * HD;
+                bulk_g2s(smem_u32(qbuf + r * Smem<HD>::kQPitch), src, HD * 2, smem_u32(&c.qfull));
             }
         }
     }
