@@ -20,10 +20,12 @@
 // TreePO (Sec. 2.3). Scores are kept in the log2 domain (q.k * log2(e)/sqrt(d))
 // so exponentials are exp2; partial LSEs are log2, the final LSE is natural.
 //
-// Pool layout. Block b holds [K|V][kv head][32 tokens][d] bf16. Inside a
-// token row the 16-byte chunk c is stored at chunk position c ^ (row & 7), so
-// that ldmatrix row gathers (8 rows, same chunk) and the CUDA-core row reads
-// (one row, 8 chunks per quarter warp) both hit 8 distinct bank groups.
+// Pool layout. Block b holds [K|V][kv head] tiles of 32 tokens x d bf16; a
+// tile is d/64 halves, each 32 rows of 128 bytes (64 elements) whose 16-byte
+// chunk c sits at position c ^ (row & 7) (see kv_off). A bulk copy of a tile
+// half lands in shared memory as 128-byte-swizzle atoms, the canonical layout
+// of tcgen05 operands, and ldmatrix row gathers (8 rows, same chunk) and
+// CUDA-core row reads both hit 8 distinct bank groups.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -130,7 +132,16 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 __device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 
-__device__ __forceinline__ int swz(int row, int chunk) { return chunk ^ (row & 7); }
+// Byte offset of 16-byte chunk `chunk` of token row `row` in a K or V tile of
+// `rows` token rows: the tile is split into 64-element halves of head_dim,
+// each half a run of 128-byte rows with chunk position (chunk & 7) ^ (row & 7)
+// -- the 128-byte-swizzle atoms (8 rows x 128 B) that tcgen05 operand
+// descriptors address, and bank-conflict free for ldmatrix row gathers and
+// for one-row reads.
+template <int ROWS>
+__device__ __forceinline__ int kv_off(int row, int chunk) {
+    return (chunk >> 3) * (ROWS * 128) + row * 128 + (((chunk & 7) ^ (row & 7)) << 4);
+}
 
 // ------------------------------------------------------------------ append --
 template <int HD>
@@ -150,7 +161,7 @@ __global__ void append_kernel(const AppendArgs a) {
         const int blk = a.blocks[pos / kBlockTokens];
         const int row = pos % kBlockTokens;
         uint8_t* dst = a.pool + (int64_t)blk * a.block_bytes + (int64_t)(kv * a.hkv + h) * a.head_bytes +
-                       row * (HD * 2) + swz(row, c) * 16;
+                       kv_off<kBlockTokens>(row, c);
         *reinterpret_cast<uint4*>(dst) = val;
     }
 }
@@ -180,7 +191,7 @@ __global__ void gather_kernel(const GatherArgs a, int64_t n_tokens) {
         const int row = (int)(tok - base);
         const int64_t blk = w >> kTileValidBits;
         const uint8_t* src = a.pool + blk * a.block_bytes + (int64_t)(kv * a.hkv + h) * a.head_bytes +
-                             row * (HD * 2) + swz(row, c) * 16;
+                             kv_off<kBlockTokens>(row, c);
         reinterpret_cast<uint4*>(kv ? a.v_out : a.k_out)[r] = *reinterpret_cast<const uint4*>(src);
     }
 }
@@ -271,12 +282,18 @@ __device__ __forceinline__ void issue_pair(const DecodeArgs& a, Ctl& c, int kvh,
     c.valid[st][0] = valid[0];
     c.valid[st][1] = valid[1];
     mbar_arrive_expect_tx(bar, bytes);  // release: the valid counts are visible to the stage's waiters
+    // a tile is HD/64 halves of 32 rows x 128 B; the stage holds each half
+    // for 64 rows, so tile j's half h lands at h * 64 * 128 + j * 32 * 128
     for (int j = 0; j < 2; ++j) {
         if (!valid[j]) continue;
         const int64_t blk = w[j] >> kTileValidBits;
         const uint8_t* src = a.pool + blk * a.block_bytes + (int64_t)kvh * a.head_bytes;
-        bulk_g2s(smem_u32(sk + j * kBlockTokens * RB), src, valid[j] * RB, bar);
-        bulk_g2s(smem_u32(sv + j * kBlockTokens * RB), src + (int64_t)a.hkv * a.head_bytes, valid[j] * RB, bar);
+#pragma unroll
+        for (int h = 0; h < HD / 64; ++h) {
+            const int so = h * kBlockTokens * 128, dofs = h * kStageTokens * 128 + j * kBlockTokens * 128;
+            bulk_g2s(smem_u32(sk + dofs), src + so, valid[j] * 128, bar);
+            bulk_g2s(smem_u32(sv + dofs), src + (int64_t)a.hkv * a.head_bytes + so, valid[j] * 128, bar);
+        }
     }
 }
 
@@ -420,7 +437,7 @@ struct CudaCorePath {
             // ---- scores: s[t][row] for this warp's TW tokens
             for (int s0 = 0; s0 < TW; s0 += TPS) {
                 const int t = tbase + s0 + ts;  // token within the stage
-                const uint4 kw = *reinterpret_cast<const uint4*>(sk + t * (HD * 2) + swz(t, dg) * 16);
+                const uint4 kw = *reinterpret_cast<const uint4*>(sk + kv_off<kStageTokens>(t, dg));
                 const uint32_t kk[4] = {kw.x, kw.y, kw.z, kw.w};
                 float kf[8];
 #pragma unroll
@@ -476,7 +493,7 @@ struct CudaCorePath {
             }
             for (int s0 = 0; s0 < TW; s0 += TPS) {
                 const int t = tbase + s0 + ts;
-                const uint4 vw = *reinterpret_cast<const uint4*>(sv + t * (HD * 2) + swz(t, dg) * 16);
+                const uint4 vw = *reinterpret_cast<const uint4*>(sv + kv_off<kStageTokens>(t, dg));
                 const uint32_t vv[4] = {vw.x, vw.y, vw.z, vw.w};
                 float vf[8];
 #pragma unroll
@@ -611,7 +628,7 @@ struct TensorPath {
                         const int tok = tbase + kb + (mi >> 1) * 8 + ri;
                         const int ch = ks * 2 + (mi & 1);
                         uint32_t b0, b1, b2, b3;
-                        ldsm_x4(sk + tok * (HD * 2) + swz(tok, ch) * 16, b0, b1, b2, b3);
+                        ldsm_x4(sk + kv_off<kStageTokens>(tok, ch), b0, b1, b2, b3);
                         mma_bf16(s[0], qa[ks], b0, b1);
                         mma_bf16(s[1], qa[ks], b2, b3);
                     }
@@ -662,7 +679,7 @@ struct TensorPath {
                         const int tok = tbase + kb + (mi & 1) * 8 + ri;
                         const int ch = dp * 2 + (mi >> 1);
                         uint32_t b0, b1, b2, b3;
-                        ldsm_x4_t(sv + tok * (HD * 2) + swz(tok, ch) * 16, b0, b1, b2, b3);
+                        ldsm_x4_t(sv + kv_off<kStageTokens>(tok, ch), b0, b1, b2, b3);
                         mma_bf16(o[2 * dp], pa, b0, b1);
                         mma_bf16(o[2 * dp + 1], pa, b2, b3);
                     }
