@@ -155,6 +155,12 @@ tp_status tp_decode(tp_tree* tree, const tp_node* leaves, int32_t n, const void*
                                       /* path (default: tensor cores, rows padded to */
                                       /* one 16-row MMA tile)                        */
 #define TP_DECODE_NO_CACHE 4u         /* rebuild the schedule even if cached         */
+#define TP_DECODE_TCGEN05 8u          /* chunks of >= 64 stacked rows and >= 32      */
+                                      /* blocks on tcgen05 (128-row units, running   */
+                                      /* concurrently with the rest)                 */
+#define TP_DECODE_ALL_TCGEN05 16u     /* every unit of > 16 stacked rows on tcgen05  */
+                                      /* Default: all stacked rows on mma.sync in    */
+                                      /* 64-row blocks (measured faster on GB300).   */
 tp_status tp_decode_ex(tp_tree* tree, const tp_node* leaves, int32_t n, const void* Q, void* O,
                        float* LSE, uint32_t flags);
 
@@ -248,9 +254,11 @@ tp_status tp_debug_gather(tp_tree* tree, tp_node leaf, void* K_out, void* V_out,
  * small; call with cap 0 to size). Layout:
  *   [0] magic 0x54505344, [1] n_units, [2] n_tiles, [3] n_occ_entries,
  *   [4] n (leaf occurrences), [5] n_slots, [6] n_merge_entries, [7] group g,
- *   [8] n_tensor_units, [9..15] reserved (0),
+ *   [8] n_mma_units, [9] n_tcgen05_units, [10..15] reserved (0),
  *   then units  [n_units][8]: tile_off, n_tiles, occ_off, row0, n_rows,
- *                             slot_base, kv_head, kind (0 CUDA-core, 1 tensor),
+ *                             slot_base, kv_head, kind (0 CUDA-core,
+ *                             1 mma.sync, 2 tcgen05); tcgen05 units first,
+ *                             then mma.sync, then CUDA-core,
  *   then tiles  [n_tiles]: block << 7 | (valid_tokens - 1),
  *   then occ    [n_occ_entries]: leaf occurrence index (row i of Q),
  *   then merge_off [n + 1], then merge_slot [n_merge_entries].

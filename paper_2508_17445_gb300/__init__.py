@@ -23,7 +23,7 @@ __all__ = [
     "tp_set_stream", "tp_add_root", "tp_append_segment", "tp_fork", "tp_prune", "tp_decode", "tp_decode_ex",
     "tp_sync", "tp_last_error", "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop",
     "tp_debug_path", "tp_debug_gather",
-    "tp_debug_schedule", "tp_decode_noalloc", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE",
+    "tp_debug_schedule", "tp_decode_noalloc", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE", "TP_DECODE_TCGEN05", "TP_DECODE_ALL_TCGEN05",
     "EXPORTED_SYMBOLS",
 ]
 
@@ -34,6 +34,8 @@ _lib: Optional[ctypes.CDLL] = None
 TP_DECODE_NO_SHARE = 1
 TP_DECODE_CUDA_CORE_SMALL = 2
 TP_DECODE_NO_CACHE = 4
+TP_DECODE_TCGEN05 = 8
+TP_DECODE_ALL_TCGEN05 = 16
 
 STATUS_NAMES = {0: "OK", -1: "INVALID_ARG", -2: "OOM", -3: "BAD_NODE", -4: "FROZEN", -5: "NOT_LEAF",
                 -6: "EMPTY_PATH", -7: "CUDA", -8: "DEVICE"}
@@ -252,7 +254,7 @@ def tp_debug_schedule(h, leaves: Sequence[int], flags: int = 0) -> Dict[str, np.
                                      buf.ctypes.data, len(buf), ctypes.byref(n_words)))
     w = buf[: n_words.value]
     assert w[0] == 0x54505344
-    n_units, n_tiles, n_occ, n, n_slots, n_merge, g, n_tensor = (int(x) for x in w[1:9])
+    n_units, n_tiles, n_occ, n, n_slots, n_merge, g, n_tensor, n_tc = (int(x) for x in w[1:10])
     off = 16
     units = w[off: off + 8 * n_units].reshape(n_units, 8)
     off += 8 * n_units
@@ -264,7 +266,7 @@ def tp_debug_schedule(h, leaves: Sequence[int], flags: int = 0) -> Dict[str, np.
     off += n + 1
     merge_slot = w[off: off + n_merge]
     return {"units": units, "tiles": tiles, "occ": occ, "merge_off": merge_off, "merge_slot": merge_slot,
-            "n_slots": n_slots, "group": g, "n_tensor_units": n_tensor, "words": w}
+            "n_slots": n_slots, "group": g, "n_tensor_units": n_tensor, "n_tc_units": n_tc, "words": w}
 
 
 # ------------------------------------------------------------------ owner --

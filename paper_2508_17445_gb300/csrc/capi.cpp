@@ -151,6 +151,9 @@ tp_status tp_tree_destroy(tp_tree* t) {
     if (t->d_part) cudaFree(t->d_part);
     if (t->d_gather_tiles) cudaFree(t->d_gather_tiles);
     for (cudaEvent_t e : t->ev_pool) cudaEventDestroy(e);
+    if (t->ev_fork) cudaEventDestroy(t->ev_fork);
+    if (t->ev_join) cudaEventDestroy(t->ev_join);
+    if (t->side) cudaStreamDestroy(t->side);
     for (int k = 0; k < 2; ++k) {
         if (t->h_pinned[k]) cudaFreeHost(t->h_pinned[k]);
         if (t->h_pinned_ev[k]) cudaEventDestroy(t->h_pinned_ev[k]);
@@ -318,6 +321,7 @@ tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void*
     a.err = t->d_err;
     a.counters = t->d_err + 1;
     a.counter = nullptr;
+    a.n_tc_units = S.n_tc;
     a.n_tensor_units = S.n_tensor;
     a.unit_begin = a.unit_end = 0;
     a.head_bytes = t->cfg.block_tokens * hd * 2;
@@ -328,9 +332,15 @@ tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void*
     a.group = hq / t->cfg.num_kv_heads;
     a.qk_scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
     cudaError_t e = cudaSuccess;
+    if (S.n_tc > 0 && S.n_units > S.n_tc && !t->side) {  // concurrent tcgen05 units need a second stream
+        e = cudaStreamCreateWithFlags(&t->side, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&t->ev_fork, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&t->ev_join, cudaEventDisableTiming);
+        if (e != cudaSuccess) return cuda_fail(t, e, "side stream");
+    }
     if (a.n_units > 0) {
         tp::LaunchTimer timer(t, tp::KK_DECODE);
-        e = tp::launch_decode(hd, a, t->stream);
+        e = tp::launch_decode(hd, a, t->stream, t->side, t->ev_fork, t->ev_join);
     }
     if (e != cudaSuccess) return cuda_fail(t, e, "decode kernel");
 
@@ -379,7 +389,7 @@ tp_status tp_decode_noalloc(tp_tree* t, const tp_node* leaves, int32_t n, const 
     float* d_part = (float*)((uint8_t*)base + sched_bytes);
     e = cudaMemcpyAsync(d_sched, S.words.data(), S.words.size() * 4, cudaMemcpyHostToDevice, t->stream);
     if (e != cudaSuccess) return cuda_fail(t, e, "schedule upload");
-    e = cudaMemsetAsync(t->d_err + 1, 0, 2 * sizeof(int32_t), t->stream);  // unit counters start at zero
+    e = cudaMemsetAsync(t->d_err + 1, 0, 3 * sizeof(int32_t), t->stream);  // unit counters start at zero
     if (e != cudaSuccess) return cuda_fail(t, e, "counter reset");
 
     tp::DecodeArgs a;
@@ -393,6 +403,7 @@ tp_status tp_decode_noalloc(tp_tree* t, const tp_node* leaves, int32_t n, const 
     a.err = t->d_err;
     a.counters = t->d_err + 1;
     a.counter = nullptr;
+    a.n_tc_units = S.n_tc;
     a.n_tensor_units = S.n_tensor;
     a.unit_begin = a.unit_end = 0;
     a.head_bytes = t->cfg.block_tokens * hd * 2;

@@ -107,6 +107,8 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     const int32_t hq = t->cfg.num_q_heads, hkv = t->cfg.num_kv_heads, g = hq / hkv;
     const bool share = !(flags & TP_DECODE_NO_SHARE);
     const bool cuda_core_small = (flags & TP_DECODE_CUDA_CORE_SMALL) != 0;
+    const bool all_tc = (flags & TP_DECODE_ALL_TCGEN05) != 0;
+    const bool use_tc = all_tc || (flags & TP_DECODE_TCGEN05) != 0;
     for (int32_t i = 0; i < n; ++i) {
         tp_status st = check_live(t, leaves[i], true);
         if (st != TP_OK) return st;
@@ -197,7 +199,7 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
         kMaxChunkTiles, std::max<int64_t>(kMinChunkTiles, (work + kTargetUnits - 1) / kTargetUnits));
 
     // 5. units, partial slots and merge entries
-    std::vector<int32_t> tensor_units, small_units;
+    std::vector<int32_t> tc_units, tensor_units, small_units;
     std::vector<int32_t> pair_occ, pair_slot;  // merge entries before sorting
     int32_t n_slots = 0;
     for (const Item& it : items) {
@@ -221,6 +223,12 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
                 if (rows < kTensorMinRows && cuda_core_small) {
                     const int32_t u[kUnitWords] = {toff, nt, it.occ_off, 0, rows, slot_base, h, KIND_CUDA_CORE};
                     small_units.insert(small_units.end(), u, u + kUnitWords);
+                } else if (use_tc && (all_tc ? rows >= kTcAnyRows : rows >= kTcMinRows && nt >= kTcMinTiles)) {
+                    for (int32_t r0 = 0; r0 < rows; r0 += kTcRowsPerUnit) {
+                        const int32_t nr = std::min(kTcRowsPerUnit, rows - r0);
+                        const int32_t u[kUnitWords] = {toff, nt, it.occ_off, r0, nr, slot_base, h, KIND_TC};
+                        tc_units.insert(tc_units.end(), u, u + kUnitWords);
+                    }
                 } else {
                     for (int32_t r0 = 0; r0 < rows; r0 += kTensorRowsPerUnit) {
                         const int32_t nr = std::min(kTensorRowsPerUnit, rows - r0);
@@ -233,7 +241,8 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
         }
     }
 
-    // 6. unit order: tensor units first, longer units first within a kind
+    // 6. unit order: tcgen05, then mma.sync, then CUDA-core units; longer
+    //    units first within a kind
     auto sort_units = [](std::vector<int32_t>& u) {
         const size_t cnt = u.size() / kUnitWords;
         std::vector<int32_t> idx(cnt);
@@ -246,6 +255,7 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
             std::memcpy(&out[k * kUnitWords], &u[(size_t)idx[k] * kUnitWords], sizeof(int32_t) * kUnitWords);
         u.swap(out);
     };
+    sort_units(tc_units);
     sort_units(tensor_units);
     sort_units(small_units);
 
@@ -259,8 +269,9 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     }
 
     // 8. assemble
+    S.n_tc = (int32_t)(tc_units.size() / kUnitWords);
     S.n_tensor = (int32_t)(tensor_units.size() / kUnitWords);
-    S.n_units = S.n_tensor + (int32_t)(small_units.size() / kUnitWords);
+    S.n_units = S.n_tc + S.n_tensor + (int32_t)(small_units.size() / kUnitWords);
     S.n_tiles = (int32_t)tiles.size();
     S.n_occ = (int32_t)occ.size();
     S.n = n;
@@ -284,8 +295,10 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     w[6] = S.n_merge;
     w[7] = g;
     w[8] = S.n_tensor;
-    std::copy(tensor_units.begin(), tensor_units.end(), w + S.off_units);
-    std::copy(small_units.begin(), small_units.end(), w + S.off_units + tensor_units.size());
+    w[9] = S.n_tc;
+    std::copy(tc_units.begin(), tc_units.end(), w + S.off_units);
+    std::copy(tensor_units.begin(), tensor_units.end(), w + S.off_units + tc_units.size());
+    std::copy(small_units.begin(), small_units.end(), w + S.off_units + tc_units.size() + tensor_units.size());
     std::copy(tiles.begin(), tiles.end(), w + S.off_tiles);
     std::copy(occ.begin(), occ.end(), w + S.off_occ);
     std::copy(merge_off.begin(), merge_off.end(), w + S.off_merge_off);

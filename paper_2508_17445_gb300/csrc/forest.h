@@ -18,14 +18,23 @@ constexpr int32_t kMaxPoolBlocks = 1 << 24;
 // Unit record: 8 int32 words (layout in treepo.h, tp_debug_schedule).
 constexpr int kUnitWords = 8;
 enum UnitWord { U_TILE_OFF, U_N_TILES, U_OCC_OFF, U_ROW0, U_N_ROWS, U_SLOT_BASE, U_KVH, U_KIND };
-enum UnitKind { KIND_CUDA_CORE = 0, KIND_TENSOR = 1 };
+enum UnitKind { KIND_CUDA_CORE = 0, KIND_TENSOR = 1, KIND_TC = 2 };
 constexpr int kSchedHeaderWords = 16;
 constexpr int32_t kSchedMagic = 0x54505344;
 // Units with fewer query rows may run on the CUDA-core path
 // (TP_DECODE_CUDA_CORE_SMALL); every other unit runs on tensor cores.
 constexpr int kTensorMinRows = 16;
-// Query rows per tensor-core unit (4 warps x one 16-row MMA tile each).
+// Query rows per mma.sync unit (4 warps x one 16-row MMA tile each).
 constexpr int kTensorRowsPerUnit = 64;
+// tcgen05 units (128 rows, MMA M) are opt-in: TP_DECODE_TCGEN05 sends chunks
+// of at least kTcMinRows stacked rows per kv head and kTcMinTiles blocks,
+// TP_DECODE_ALL_TCGEN05 every unit of more than one 16-row MMA tile. By
+// default every unit runs on mma.sync, which measured faster on GB300: the
+// tcgen05 pipeline pays a longer start and drain per unit.
+constexpr int kTcMinRows = 64;
+constexpr int kTcMinTiles = 32;
+constexpr int kTcAnyRows = 17;
+constexpr int kTcRowsPerUnit = 128;
 // Longest unit in pool blocks (the decode kernel keeps a unit's tile words
 // in shared memory).
 constexpr int kMaxUnitTiles = 128;
@@ -44,9 +53,10 @@ struct DecodeArgs {
     float* part_o;      // [slot][Hq][hd], normalised partial output
     float* part_lse;    // [slot][Hq], log2-domain partial LSE
     int32_t* err;
-    int32_t* counters;    // [2] next unit per kind (0 at launch; the merge re-arms them)
+    int32_t* counters;    // [3] next unit per kind (0 at launch; the merge re-arms them)
     int32_t* counter;     // the counter of the launch in flight (set by the launcher)
-    int32_t n_tensor_units;  // units [0, n_tensor_units) are tensor units
+    int32_t n_tc_units;      // units [0, n_tc) are tcgen05 units,
+    int32_t n_tensor_units;  // then n_tensor mma.sync units, then CUDA-core units
     int32_t unit_begin, unit_end;  // unit range of the launch in flight
     int64_t block_bytes;  // bytes of one pool block (K and V, all kv heads)
     int32_t head_bytes;   // bytes of one (block, K|V, kv head) tile
@@ -64,7 +74,7 @@ struct MergeArgs {
     const float* part_lse;
     uint16_t* out;  // bf16 [n][Hq][hd]
     float* lse;     // [n][Hq], natural log
-    int32_t* counters;  // decode's two unit counters, reset to 0 here
+    int32_t* counters;  // decode's three unit counters, reset to 0 here
     int32_t n;
     int32_t hq;
 };
@@ -95,7 +105,11 @@ struct GatherArgs {
 
 // Launchers (kernels.cu). Return cudaSuccess or the launch error.
 cudaError_t launch_append(int head_dim, const AppendArgs& a, cudaStream_t s);
-cudaError_t launch_decode(int head_dim, const DecodeArgs& a, cudaStream_t s);
+// With side != nullptr and both tcgen05 and other units present, the
+// tcgen05 units run on `side` concurrently with the rest (fork/join through
+// the two events), so a small tcgen05 launch does not leave SMs idle.
+cudaError_t launch_decode(int head_dim, const DecodeArgs& a, cudaStream_t s, cudaStream_t side = nullptr,
+                          cudaEvent_t fork = nullptr, cudaEvent_t join = nullptr);
 cudaError_t launch_merge(int head_dim, const MergeArgs& a, cudaStream_t s);
 cudaError_t launch_gather(int head_dim, const GatherArgs& a, int64_t n_tokens, cudaStream_t s);
 int decode_smem_bytes(int head_dim);
@@ -129,7 +143,7 @@ class BlockPool {
 
 struct Schedule {
     std::vector<int32_t> words;  // header | units | tiles | occ | merge_off | merge_slot
-    int32_t n_units = 0, n_tiles = 0, n_occ = 0, n = 0, n_slots = 0, n_merge = 0, n_tensor = 0;
+    int32_t n_units = 0, n_tiles = 0, n_occ = 0, n = 0, n_slots = 0, n_merge = 0, n_tensor = 0, n_tc = 0;
     int64_t off_units = 0, off_tiles = 0, off_occ = 0, off_merge_off = 0, off_merge_slot = 0;
 };
 
@@ -150,7 +164,7 @@ struct tp_tree {
     uint32_t epoch = 0;
 
     // device scratch owned by the library
-    int32_t* d_err = nullptr;  // [0] device error flag, [1..2] decode unit counters
+    int32_t* d_err = nullptr;  // [0] device error flag, [1..3] decode unit counters
     int32_t* d_sched = nullptr;
     int64_t d_sched_cap = 0;  // words
     float* d_part = nullptr;  // partial o then partial lse
@@ -161,6 +175,8 @@ struct tp_tree {
     int pinned_next = 0;
     int32_t* d_gather_tiles = nullptr;
     int64_t d_gather_cap = 0;
+    cudaStream_t side = nullptr;  // second stream for concurrent tcgen05 units
+    cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
 
     // kernel timing (tp_profile_start / tp_profile_stop)
     bool profiling = false;

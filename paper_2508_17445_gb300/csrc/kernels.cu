@@ -76,6 +76,17 @@ __device__ __forceinline__ float fast_exp2(float x) {  // ex2.approx: exp2(-inf)
     return y;
 }
 
+// Non-blocking probe of an mbarrier phase.
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
 __device__ __forceinline__ uint64_t global_ns() {
     uint64_t t;
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
@@ -257,7 +268,8 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
-__device__ __forceinline__ void note_timeout(const DecodeArgs& a, Ctl& c, int code) {
+template <typename CtlT>
+__device__ __forceinline__ void note_timeout(const DecodeArgs& a, CtlT& c, int code) {
     atomicOr(a.err, code);
     *reinterpret_cast<volatile int*>(&c.abort) = 1;
 }
@@ -265,8 +277,8 @@ __device__ __forceinline__ void note_timeout(const DecodeArgs& a, Ctl& c, int co
 // Producer: issue the bulk copies of one tile pair (tile words w[0..1],
 // w = -1 for a missing second tile) into stage `st`, and record the pair's
 // valid token counts for the consumers.
-template <int HD>
-__device__ __forceinline__ void issue_pair(const DecodeArgs& a, Ctl& c, int kvh, uint8_t* ring, const int32_t (&w)[2],
+template <int HD, typename CtlT>
+__device__ __forceinline__ void issue_pair(const DecodeArgs& a, CtlT& c, int kvh, uint8_t* ring, const int32_t (&w)[2],
                                            int st) {
     constexpr int RB = HD * 2;
     uint8_t* sk = ring + st * Smem<HD>::kStageBytes;
@@ -925,13 +937,567 @@ __global__ void __launch_bounds__(kDecodeThreads, 2) decode_kernel(const DecodeA
     consume<HD, KIND>(a, ctl, ring, park, qbuf, cc_scratch);
 }
 
+
+// ---------------------------------------------------------- tcgen05 path --
+// Units of 17..128 stacked query rows: Q.K^T and P.V run as tcgen05.mma
+// (M = 128 rows, bf16 -> fp32) issued by one thread, accumulators in tensor
+// memory. Warps: 0-3 softmax + epilogue (warp w owns TMEM lanes 32w..32w+31,
+// i.e. query rows 32w..32w+31: one row per thread, no shuffles), 4 the K/V
+// streamer, 5 the unit fetcher (also stages the unit's query rows in the
+// swizzled operand layout), 6 the MMA issuer.
+//   S = Q K^T    A = query rows (smem, K-major), B = K stage (smem, K-major),
+//                D = S buffer (TMEM, 64 columns, double-buffered)
+//   O += P V     A = P (TMEM, bf16 pairs written over the S buffer),
+//                B = V stage (smem, MN-major), D = O (TMEM, HD columns)
+// S of the next stage is issued before P.V of the current one, so the
+// tensor core overlaps the softmax. O is rescaled only when a row's running
+// max grows by more than 2^8 (p <= 256 stays exact in fp32 and ~bf16);
+// otherwise the stale max is kept, which leaves O / l unchanged.
+constexpr int kTcConsumerWarps = 4;
+constexpr int kTcStreamerWarp = 4, kTcFetcherWarp = 5, kTcIssuerWarp = 6;
+constexpr int kTcThreads = 7 * 32;
+constexpr int kTcRows = 128;          // MMA M (unit rows padded to it)
+constexpr uint32_t kTmemCols = 256;   // S0 [0,64) S1 [64,128) O [128, 128 + HD)
+constexpr float kRescaleLog2 = 8.f;
+
+template <int HD>
+struct TcSmem {
+    static constexpr int kStageBytes = 2 * (HD / 64) * kStageTokens * 128;  // K then V of 64 tokens
+    static constexpr int kRingBytes = kStages * kStageBytes;
+    static constexpr int kQBytes = (HD / 64) * kTcRows * 128;
+    static constexpr int kBytes = kRingBytes + kQBytes + 1024;  // + slack to align to 1024
+};
+
+struct CtlTc {
+    uint64_t kfull[kStages];   // K half of the stage landed (streamer + TMA bytes)
+    uint64_t kempty[kStages];  // K half read by Q.K^T (issuer's commit)
+    uint64_t vfull[kStages];   // V half landed
+    uint64_t vempty[kStages];  // V half read by P.V (issuer's commit)
+    uint64_t ufull[2], uempty[2];
+    uint64_t qfull;           // query rows staged (fetcher)
+    uint64_t qempty;          // the unit's last Q.K^T done (issuer's commit)
+    uint64_t s_full[2];       // S buffer holds scores (issuer's commit)
+    uint64_t p_full[2];       // S buffer holds P (one arrival per consumer warp)
+    uint64_t o_full;          // the unit's last P.V done (issuer's commit)
+    uint64_t o_free;          // the epilogue has read O (one arrival per consumer warp)
+    uint64_t pv_done;         // a P.V finished (issuer's commit; rescale waits)
+    int valid[kStages][2];
+    int unit[2];
+    int desc[2][kUnitWords];
+    int tiles[2][kMaxUnitTiles];
+    int64_t qrow[kTcRows];    // element offset in Q of each row being staged
+    uint32_t tmem;
+    int abort;
+};
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+
+// sm_100 shared-memory matrix descriptor: 128-byte swizzle, version 1.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    return (uint64_t)((saddr >> 4) & 0x3FFF) | ((uint64_t)((lbo >> 4) & 0x3FFF) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3FFF) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, M = 128.
+template <int N, bool B_MN_MAJOR>
+__device__ __forceinline__ constexpr uint32_t mma_idesc() {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((B_MN_MAJOR ? 1u : 0u) << 16) | ((uint32_t)(N >> 3) << 17) |
+           ((uint32_t)(kTcRows >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_ss(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{ .reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p; }" ::"r"(d),
+        "l"(a), "l"(b), "r"(idesc), "r"(acc));
+}
+
+__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{ .reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p; }" ::"r"(d),
+        "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc));
+}
+
+// 32 consecutive TMEM columns of this thread's lane
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
+        "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+          "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,"
+        "%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+        "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]),
+        "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]),
+        "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ UnitDesc read_desc(const int* slot) {
+    const volatile int* dw = slot;
+    UnitDesc d;
+    d.tile_off = dw[U_TILE_OFF];
+    d.n_tiles = dw[U_N_TILES];
+    d.occ_off = dw[U_OCC_OFF];
+    d.row0 = dw[U_ROW0];
+    d.n_rows = dw[U_N_ROWS];
+    d.slot_base = dw[U_SLOT_BASE];
+    d.kvh = dw[U_KVH];
+    d.kind = dw[U_KIND];
+    return d;
+}
+
+// Fetcher warp: claim units, publish descriptor + tile words, stage query rows
+// in the 128-byte-swizzle K-major layout the MMA reads. Rows past n_rows are
+// left as they are: a row of A only reaches the same row of S, P and O, and
+// those rows are never written out.
+template <int HD>
+__device__ void tc_fetch(const DecodeArgs& a, CtlTc& c, uint8_t* qbuf) {
+    const int lane = threadIdx.x & 31;
+    volatile int* abort = &c.abort;
+    for (int k = 0;; ++k) {
+        const int q = k & 1;
+        if (!mbar_wait(smem_u32(&c.uempty[q]), ((k >> 1) & 1) ^ 1)) note_timeout(a, c, 2);
+        int u = -1;
+        if (lane == 0) {
+            u = *abort ? -1 : a.unit_begin + atomicAdd(a.counter, 1);
+            if (u >= a.unit_end) u = -1;
+        }
+        u = __shfl_sync(0xffffffffu, u, 0);
+        const int word = (u >= 0 && lane < kUnitWords) ? a.units[(int64_t)u * kUnitWords + lane] : 0;
+        const int n_tiles = __shfl_sync(0xffffffffu, word, U_N_TILES);
+        const int tile_off = __shfl_sync(0xffffffffu, word, U_TILE_OFF);
+        if (u >= 0)
+            for (int t = lane; t < n_tiles; t += 32) c.tiles[q][t] = a.tiles[tile_off + t];
+        if (lane < kUnitWords) reinterpret_cast<volatile int*>(c.desc[q])[lane] = word;
+        if (lane == 0) *reinterpret_cast<volatile int*>(&c.unit[q]) = u;
+        __threadfence_block();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&c.ufull[q]));
+        if (u < 0) return;
+        const int occ_off = __shfl_sync(0xffffffffu, word, U_OCC_OFF);
+        const int row0 = __shfl_sync(0xffffffffu, word, U_ROW0);
+        const int n_rows = __shfl_sync(0xffffffffu, word, U_N_ROWS);
+        const int kvh = __shfl_sync(0xffffffffu, word, U_KVH);
+        // the previous unit's Q.K^T MMAs have read the buffer
+        if (!mbar_wait(smem_u32(&c.qempty), (k & 1) ^ 1)) note_timeout(a, c, 2);
+        constexpr int CH = HD / 8;  // 16-byte chunks per row
+        constexpr int BATCH = 16;   // loads in flight per lane
+        const int g = a.group;
+        for (int r = lane; r < n_rows; r += 32) {  // row pointers: one round trip
+            const int item_row = row0 + r;
+            c.qrow[r] = ((int64_t)a.occ[occ_off + item_row / g] * a.hq + kvh * g + item_row % g) * HD;
+        }
+        __syncwarp();
+        const int total = n_rows * CH;
+        for (int base = 0; base < total; base += 32 * BATCH) {
+            uint4 v[BATCH];
+#pragma unroll
+            for (int b = 0; b < BATCH; ++b) {
+                const int idx = base + b * 32 + lane;
+                if (idx < total) v[b] = *reinterpret_cast<const uint4*>(a.q + c.qrow[idx / CH] + (idx % CH) * 8);
+            }
+#pragma unroll
+            for (int b = 0; b < BATCH; ++b) {
+                const int idx = base + b * 32 + lane;
+                if (idx < total) *reinterpret_cast<uint4*>(qbuf + kv_off<kTcRows>(idx / CH, idx % CH)) = v[b];
+            }
+        }
+        fence_proxy_async();  // generic stores -> visible to the tensor core
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&c.qfull));
+    }
+}
+
+// Bulk copies of one half (K or V) of a tile pair into a stage; w = -1 for a
+// missing second tile.
+template <int HD>
+__device__ __forceinline__ void issue_half(const DecodeArgs& a, int kvh, int kv, uint8_t* dst, const int32_t (&w)[2],
+                                           uint32_t bar) {
+    uint32_t bytes = 0;
+    int valid[2] = {0, 0};
+    for (int j = 0; j < 2; ++j)
+        if (w[j] >= 0) {
+            valid[j] = (w[j] & ((1 << kTileValidBits) - 1)) + 1;
+            bytes += (uint32_t)(valid[j] * HD * 2);
+        }
+    mbar_arrive_expect_tx(bar, bytes);
+    for (int j = 0; j < 2; ++j) {
+        if (!valid[j]) continue;
+        const uint8_t* src = a.pool + (int64_t)(w[j] >> kTileValidBits) * a.block_bytes +
+                             (int64_t)(kv * a.hkv + kvh) * a.head_bytes;
+#pragma unroll
+        for (int h = 0; h < HD / 64; ++h)
+            bulk_g2s(smem_u32(dst + h * kStageTokens * 128 + j * kBlockTokens * 128), src + h * kBlockTokens * 128,
+                     valid[j] * 128, bar);
+    }
+}
+
+// Streamer lane: K and V halves of each published unit's tile pairs, each
+// half refilled as soon as its own slot frees (K is freed by Q.K^T, V only by
+// P.V, so K runs ahead while V waits for the softmax).
+template <int HD>
+__device__ void tc_stream(const DecodeArgs& a, CtlTc& c, uint8_t* ring) {
+    int ks = 0, vs = 0;
+    uint32_t kph = 0, vph = 0;
+    for (int k = 0;; ++k) {
+        const int q = k & 1;
+        if (!mbar_wait(smem_u32(&c.ufull[q]), (k >> 1) & 1)) {
+            note_timeout(a, c, 2);
+            return;
+        }
+        if (*reinterpret_cast<volatile int*>(&c.unit[q]) < 0) return;
+        const int n_tiles = *reinterpret_cast<volatile int*>(&c.desc[q][U_N_TILES]);
+        const int kvh = *reinterpret_cast<volatile int*>(&c.desc[q][U_KVH]);
+        const volatile int* tw = c.tiles[q];
+        const int n_pairs = (n_tiles + 1) / 2;
+        int kj = 0, vj = 0;
+        uint64_t idle_since = 0;
+        uint32_t spins = 0;
+        while (vj < n_pairs) {
+            bool progress = false;
+            if (kj < n_pairs && mbar_test(smem_u32(&c.kempty[ks]), kph ^ 1)) {
+                const int32_t w[2] = {tw[2 * kj], 2 * kj + 1 < n_tiles ? tw[2 * kj + 1] : -1};
+                fence_proxy_async();
+                issue_half<HD>(a, kvh, 0, ring + ks * TcSmem<HD>::kStageBytes, w, smem_u32(&c.kfull[ks]));
+                if (++ks == kStages) {
+                    ks = 0;
+                    kph ^= 1;
+                }
+                ++kj;
+                progress = true;
+            }
+            if (vj < kj && mbar_test(smem_u32(&c.vempty[vs]), vph ^ 1)) {
+                const int32_t w[2] = {tw[2 * vj], 2 * vj + 1 < n_tiles ? tw[2 * vj + 1] : -1};
+                fence_proxy_async();
+                issue_half<HD>(a, kvh, 1, ring + vs * TcSmem<HD>::kStageBytes + (HD / 64) * kStageTokens * 128, w,
+                               smem_u32(&c.vfull[vs]));
+                if (++vs == kStages) {
+                    vs = 0;
+                    vph ^= 1;
+                }
+                ++vj;
+                progress = true;
+            }
+            if (progress) {
+                spins = 0;
+                idle_since = 0;
+            } else if ((++spins & 1023) == 0) {
+                const uint64_t now = global_ns();
+                if (idle_since == 0) {
+                    idle_since = now;
+                } else if (now - idle_since > kWaitLimitNs) {
+                    note_timeout(a, c, 2);
+                    return;
+                }
+            }
+        }
+        mbar_arrive(smem_u32(&c.uempty[q]));
+    }
+}
+
+// MMA issuer lane.
+template <int HD>
+__device__ void tc_issue(const DecodeArgs& a, CtlTc& c, const uint8_t* ring, const uint8_t* qbuf) {
+    constexpr uint32_t kIdescS = mma_idesc<kStageTokens, false>();
+    constexpr uint32_t kIdescPV = mma_idesc<HD, true>();
+    const uint32_t tmem = c.tmem;
+    const uint32_t q_addr = smem_u32(qbuf), ring_addr = smem_u32(ring);
+    int s_stage = 0, v_stage = 0;
+    uint32_t s_phase = 0, v_phase = 0;
+    uint32_t gs = 0;  // stages issued by this CTA so far (S buffer = gs & 1)
+    for (int k = 0;; ++k) {
+        const int q = k & 1;
+        if (!mbar_wait(smem_u32(&c.ufull[q]), (k >> 1) & 1)) {
+            note_timeout(a, c, 2);
+            return;
+        }
+        if (*reinterpret_cast<volatile int*>(&c.unit[q]) < 0) return;
+        const int n_tiles = *reinterpret_cast<volatile int*>(&c.desc[q][U_N_TILES]);
+        const int n_pairs = (n_tiles + 1) / 2;
+        if (!mbar_wait(smem_u32(&c.qfull), k & 1)) note_timeout(a, c, 2);
+        tc_fence_after();
+        // Event loop: issue Q.K^T of the next stage as soon as its K/V has
+        // landed (and its S buffer is free, i.e. P.V two stages back is
+        // issued), and P.V of the oldest stage as soon as its P is written;
+        // neither waits on the other.
+        int next_s = 0, next_pv = 0;
+        bool q_released = false;
+        uint64_t idle_since = 0;
+        uint32_t spins = 0;
+        while (next_pv < n_pairs) {
+            bool progress = false;
+            if (next_s < n_pairs && next_s <= next_pv + 1 && mbar_test(smem_u32(&c.kfull[s_stage]), s_phase)) {
+                tc_fence_after();
+                const uint32_t g_stage = gs + next_s;
+                const uint32_t kb = ring_addr + s_stage * TcSmem<HD>::kStageBytes;
+                const uint32_t d = tmem + (g_stage & 1) * kStageTokens;
+#pragma unroll
+                for (int ks = 0; ks < HD / 16; ++ks) {
+                    const uint32_t off = (ks >> 2) * (kStageTokens * 128) + (ks & 3) * 32;
+                    const uint32_t qoff = (ks >> 2) * (kTcRows * 128) + (ks & 3) * 32;
+                    mma_ss(d, smem_desc(q_addr + qoff, 16, 1024), smem_desc(kb + off, 16, 1024), kIdescS, ks > 0);
+                }
+                tc_commit(smem_u32(&c.s_full[g_stage & 1]));
+                tc_commit(smem_u32(&c.kempty[s_stage]));
+                if (++s_stage == kStages) {
+                    s_stage = 0;
+                    s_phase ^= 1;
+                }
+                ++next_s;
+                progress = true;
+            }
+            if (next_s == n_pairs && !q_released) {
+                tc_commit(smem_u32(&c.qempty));  // every Q.K^T of the unit issued
+                q_released = true;
+            }
+            const uint32_t gp = gs + next_pv;
+            if (next_pv < next_s && mbar_test(smem_u32(&c.p_full[gp & 1]), (gp >> 1) & 1) &&
+                mbar_test(smem_u32(&c.vfull[v_stage]), v_phase)) {
+                tc_fence_after();
+                if (next_pv == 0) {  // the previous unit's epilogue has read O
+                    if (!mbar_wait(smem_u32(&c.o_free), (k & 1) ^ 1)) note_timeout(a, c, 2);
+                    tc_fence_after();
+                }
+                const uint32_t vb = ring_addr + v_stage * TcSmem<HD>::kStageBytes + (HD / 64) * kStageTokens * 128;
+                const uint32_t p_tmem = tmem + (gp & 1) * kStageTokens;
+#pragma unroll
+                for (int kk = 0; kk < kStageTokens / 16; ++kk)
+                    mma_ts(tmem + 2 * kStageTokens, p_tmem + kk * 8,
+                           smem_desc(vb + kk * 2048, kStageTokens * 128, 1024), kIdescPV,
+                           (next_pv > 0 || kk > 0) ? 1u : 0u);
+                tc_commit(smem_u32(&c.vempty[v_stage]));
+                tc_commit(smem_u32(&c.pv_done));
+                if (next_pv + 1 == n_pairs) tc_commit(smem_u32(&c.o_full));
+                if (++v_stage == kStages) {
+                    v_stage = 0;
+                    v_phase ^= 1;
+                }
+                ++next_pv;
+                progress = true;
+            }
+            if (progress) {
+                spins = 0;
+                idle_since = 0;
+            } else if ((++spins & 1023) == 0) {  // bounded: give up after the wait limit
+                const uint64_t now = global_ns();
+                if (idle_since == 0) {
+                    idle_since = now;
+                } else if (now - idle_since > kWaitLimitNs) {
+                    note_timeout(a, c, 2);
+                    return;
+                }
+            }
+        }
+        gs += n_pairs;
+        mbar_arrive(smem_u32(&c.uempty[q]));
+    }
+}
+
+// Softmax + epilogue warps: thread = query row (warp * 32 + lane).
+template <int HD>
+__device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int row = warp * 32 + lane;
+    const uint32_t lane_addr = c.tmem + ((uint32_t)(warp * 32) << 16);
+    const uint32_t o_addr = lane_addr + 2 * kStageTokens;
+    uint32_t gs = 0;
+    for (int k = 0;; ++k) {
+        const int q = k & 1;
+        if (!mbar_wait(smem_u32(&c.ufull[q]), (k >> 1) & 1)) {
+            note_timeout(a, c, 8);
+            return;
+        }
+        if (*reinterpret_cast<volatile int*>(&c.unit[q]) < 0) return;
+        const UnitDesc d = read_desc(c.desc[q]);
+        const volatile int* tw = c.tiles[q];
+        const int n_pairs = (d.n_tiles + 1) / 2;
+        float m_used = -INFINITY, l = 0.f;
+        for (int j = 0; j < n_pairs; ++j) {
+            const uint32_t g_stage = gs + j, sb = g_stage & 1;
+            const int v0 = (tw[2 * j] & ((1 << kTileValidBits) - 1)) + 1;
+            const int v1 = 2 * j + 1 < d.n_tiles ? (tw[2 * j + 1] & ((1 << kTileValidBits) - 1)) + 1 : 0;
+            if (!mbar_wait(smem_u32(&c.s_full[sb]), (g_stage >> 1) & 1)) note_timeout(a, c, 1);
+            tc_fence_after();
+            if (warp * 32 >= d.n_rows) {  // padding rows only: their P is never read back
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&c.p_full[sb]));
+                continue;
+            }
+            const uint32_t s_addr = lane_addr + sb * kStageTokens;
+            uint32_t r[32];
+            // pass 1: row max over the stage's valid tokens
+            float mx = -INFINITY;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                tmem_ld32(s_addr + h * 32, r);
+                const int lim = h ? v1 : v0;
+#pragma unroll
+                for (int t = 0; t < 32; ++t)
+                    if (t < lim) mx = fmaxf(mx, __uint_as_float(r[t]) * a.qk_scale_log2);
+            }
+            const float m_new = fmaxf(m_used, mx);
+            const bool need = m_new > m_used + kRescaleLog2;
+            if (__any_sync(0xffffffffu, need)) {
+                const float alpha = need ? fast_exp2(m_used - m_new) : 1.f;
+                if (j > 0) {  // O holds earlier stages: wait for the last P.V, then scale it
+                    if (!mbar_wait(smem_u32(&c.pv_done), (g_stage - 1) & 1)) note_timeout(a, c, 1);
+                    tc_fence_after();
+#pragma unroll 1
+                    for (int cc = 0; cc < HD / 32; ++cc) {
+                        uint32_t ov[32];
+                        tmem_ld32(o_addr + cc * 32, ov);
+#pragma unroll
+                        for (int t = 0; t < 32; ++t) ov[t] = __float_as_uint(__uint_as_float(ov[t]) * alpha);
+                        tmem_st32(o_addr + cc * 32, ov);
+                    }
+                }
+                if (need) {
+                    l *= alpha;
+                    m_used = m_new;
+                }
+            }
+            // pass 2: P = exp2(s - m_used) as bf16 pairs over the S columns
+            uint32_t pw[32];
+            float sum = 0.f;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                tmem_ld32(s_addr + h * 32, r);
+                const int lim = h ? v1 : v0;
+#pragma unroll
+                for (int t = 0; t < 32; t += 2) {
+                    const float p0 = t < lim ? fast_exp2(__uint_as_float(r[t]) * a.qk_scale_log2 - m_used) : 0.f;
+                    const float p1 = t + 1 < lim ? fast_exp2(__uint_as_float(r[t + 1]) * a.qk_scale_log2 - m_used) : 0.f;
+                    sum += p0 + p1;
+                    pw[h * 16 + t / 2] = pack_bf16(p0, p1);
+                }
+            }
+            l += sum;
+            tmem_st32(s_addr, pw);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&c.p_full[sb]));
+        }
+        gs += n_pairs;
+        // epilogue: O / l and the log2 LSE of this row
+        if (!mbar_wait(smem_u32(&c.o_full), k & 1)) note_timeout(a, c, 1);
+        tc_fence_after();
+        if (warp * 32 >= d.n_rows) {  // padding rows only
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(smem_u32(&c.o_free));
+                mbar_arrive(smem_u32(&c.uempty[q]));
+            }
+            continue;
+        }
+        const bool live = row < d.n_rows;
+        float* dst = nullptr;
+        if (live) {
+            const int item_row = d.row0 + row;
+            const int slot = d.slot_base + item_row / a.group;
+            const int qh = d.kvh * a.group + item_row % a.group;
+            dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
+            a.part_lse[(int64_t)slot * a.hq + qh] = m_used + __log2f(l);
+        }
+        const float inv = 1.f / l;
+#pragma unroll 1
+        for (int cc = 0; cc < HD / 32; ++cc) {
+            uint32_t ov[32];
+            tmem_ld32(o_addr + cc * 32, ov);
+            if (live)
+#pragma unroll
+                for (int t = 0; t < 32; t += 4)
+                    *reinterpret_cast<float4*>(dst + cc * 32 + t) =
+                        make_float4(__uint_as_float(ov[t]) * inv, __uint_as_float(ov[t + 1]) * inv,
+                                    __uint_as_float(ov[t + 2]) * inv, __uint_as_float(ov[t + 3]) * inv);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+            mbar_arrive(smem_u32(&c.o_free));
+            mbar_arrive(smem_u32(&c.uempty[q]));
+        }
+    }
+}
+
+template <int HD>
+__global__ void __launch_bounds__(kTcThreads, 2) decode_tc_kernel(const DecodeArgs a) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    __shared__ __align__(16) CtlTc ctl;
+    // 128-byte-swizzle operands need 1024-byte-aligned atoms
+    uint8_t* base = smem_raw + ((1024 - (smem_u32(smem_raw) & 1023)) & 1023);
+    uint8_t* ring = base;
+    uint8_t* qbuf = base + TcSmem<HD>::kRingBytes;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    {
+        uint4* r4 = reinterpret_cast<uint4*>(ring);  // rows past a partial block must be finite
+        for (int i = tid; i < TcSmem<HD>::kRingBytes / 16; i += kTcThreads) r4[i] = make_uint4(0, 0, 0, 0);
+    }
+    if (tid == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(smem_u32(&ctl.kfull[s]), 1);
+            mbar_init(smem_u32(&ctl.kempty[s]), 1);
+            mbar_init(smem_u32(&ctl.vfull[s]), 1);
+            mbar_init(smem_u32(&ctl.vempty[s]), 1);
+        }
+        for (int q = 0; q < 2; ++q) {
+            mbar_init(smem_u32(&ctl.ufull[q]), 1);
+            mbar_init(smem_u32(&ctl.uempty[q]), kTcConsumerWarps + 2);  // consumers + streamer + issuer
+            mbar_init(smem_u32(&ctl.s_full[q]), 1);
+            mbar_init(smem_u32(&ctl.p_full[q]), kTcConsumerWarps);
+        }
+        mbar_init(smem_u32(&ctl.qfull), 1);
+        mbar_init(smem_u32(&ctl.qempty), 1);
+        mbar_init(smem_u32(&ctl.o_full), 1);
+        mbar_init(smem_u32(&ctl.o_free), kTcConsumerWarps);
+        mbar_init(smem_u32(&ctl.pv_done), 1);
+        ctl.abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&ctl.tmem)),
+                     "r"(kTmemCols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    fence_proxy_async();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp < kTcConsumerWarps)
+        tc_consume<HD>(a, ctl);
+    else if (warp == kTcStreamerWarp) {
+        if ((tid & 31) == 0) tc_stream<HD>(a, ctl, ring);
+    } else if (warp == kTcFetcherWarp)
+        tc_fetch<HD>(a, ctl, qbuf);
+    else if ((tid & 31) == 0)
+        tc_issue<HD>(a, ctl, ring, qbuf);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(ctl.tmem), "r"(kTmemCols));
+}
+
 // ------------------------------------------------------------------- merge --
 template <int HD>
 __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
     constexpr int DPL = HD / 32;  // dims per lane: 4 or 2
     const int warp_global = blockIdx.x * 4 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
-    if (blockIdx.x == 0 && threadIdx.x < 2) a.counters[threadIdx.x] = 0;  // decode is done: re-arm its counters
+    if (blockIdx.x == 0 && threadIdx.x < 3) a.counters[threadIdx.x] = 0;  // decode is done: re-arm its counters
     if (warp_global >= a.n * a.hq) return;
     const int i = warp_global / a.hq, qh = warp_global % a.hq;
     const int beg = a.merge_off[i], end = a.merge_off[i + 1];
@@ -1002,10 +1568,55 @@ cudaError_t launch_range(DecodeArgs a, int begin, int end, int32_t* counter, cud
 }
 
 template <int HD>
-cudaError_t launch_decode_hd(const DecodeArgs& a, cudaStream_t s) {
-    cudaError_t e = launch_range<HD, KIND_TENSOR>(a, 0, a.n_tensor_units, a.counters, s);
+int decode_tc_grid() {
+    static int grid = [] {
+        int dev = 0, sms = 0, per_sm = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (cudaFuncSetAttribute(decode_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 TcSmem<HD>::kBytes) != cudaSuccess)
+            return 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_tc_kernel<HD>, kTcThreads,
+                                                          TcSmem<HD>::kBytes) != cudaSuccess)
+            return 0;
+        // each resident CTA holds kTmemCols of the SM's 512 tensor-memory columns
+        return sms * std::min(std::max(per_sm, 1), 512 / (int)kTmemCols);
+    }();
+    return grid;
+}
+
+template <int HD>
+cudaError_t launch_tc_range(DecodeArgs a, int begin, int end, int32_t* counter, cudaStream_t s) {
+    if (end <= begin) return cudaSuccess;
+    const int slots = decode_tc_grid<HD>();
+    if (slots == 0) return cudaErrorInvalidConfiguration;
+    a.unit_begin = begin;
+    a.unit_end = end;
+    a.counter = counter;
+    decode_tc_kernel<HD><<<std::min(end - begin, slots), kTcThreads, TcSmem<HD>::kBytes, s>>>(a);
+    return cudaGetLastError();
+}
+
+template <int HD>
+cudaError_t launch_decode_hd(const DecodeArgs& a, cudaStream_t s, cudaStream_t side, cudaEvent_t fork,
+                             cudaEvent_t join) {
+    const int tc_end = a.n_tc_units, mma_end = tc_end + a.n_tensor_units;
+    cudaError_t e;
+    const bool concurrent = side && fork && join && tc_end > 0 && a.n_units > tc_end;
+    if (concurrent) {
+        if ((e = cudaEventRecord(fork, s)) != cudaSuccess) return e;
+        if ((e = cudaStreamWaitEvent(side, fork, 0)) != cudaSuccess) return e;
+        if ((e = launch_tc_range<HD>(a, 0, tc_end, a.counters, side)) != cudaSuccess) return e;
+        if ((e = cudaEventRecord(join, side)) != cudaSuccess) return e;
+    } else {
+        e = launch_tc_range<HD>(a, 0, tc_end, a.counters, s);
+    }
     if (e != cudaSuccess) return e;
-    return launch_range<HD, KIND_CUDA_CORE>(a, a.n_tensor_units, a.n_units, a.counters + 1, s);
+    e = launch_range<HD, KIND_TENSOR>(a, tc_end, mma_end, a.counters + 1, s);
+    if (e != cudaSuccess) return e;
+    e = launch_range<HD, KIND_CUDA_CORE>(a, mma_end, a.n_units, a.counters + 2, s);
+    if (e != cudaSuccess) return e;
+    return concurrent ? cudaStreamWaitEvent(s, join, 0) : cudaSuccess;
 }
 
 }  // namespace
@@ -1059,9 +1670,10 @@ cudaError_t launch_gather(int hd, const GatherArgs& a, int64_t n_tokens, cudaStr
     return cudaGetLastError();
 }
 
-cudaError_t launch_decode(int hd, const DecodeArgs& a, cudaStream_t s) {
+cudaError_t launch_decode(int hd, const DecodeArgs& a, cudaStream_t s, cudaStream_t side, cudaEvent_t fork,
+                          cudaEvent_t join) {
     if (a.n_units == 0) return cudaSuccess;
-    return hd == 64 ? launch_decode_hd<64>(a, s) : launch_decode_hd<128>(a, s);
+    return hd == 64 ? launch_decode_hd<64>(a, s, side, fork, join) : launch_decode_hd<128>(a, s, side, fork, join);
 }
 
 cudaError_t launch_merge(int hd, const MergeArgs& a, cudaStream_t s) {

@@ -266,12 +266,22 @@ def check_schedule(f, ids, model, script, leaves_sid, flags=0):
     for u in S["units"]:
         toff, nt, ooff, row0, nrows, sbase, kvh, kind = (int(x) for x in u)
         assert 0 <= kvh < heads.num_kv_heads
-        if kind == 0:
+        if kind == 0:                      # CUDA-core: one leaf group, < 16 rows
             assert nrows < 16 and flags & tp.TP_DECODE_CUDA_CORE_SMALL
-        else:
-            assert 1 <= nrows <= 64
+        elif kind == 1:                    # mma.sync: 64-row blocks (<= 16 rows with all-tcgen05)
+            if flags & tp.TP_DECODE_ALL_TCGEN05:
+                assert row0 == 0 and 1 <= nrows <= 16
+            else:
+                assert 1 <= nrows <= 64
             if flags & tp.TP_DECODE_CUDA_CORE_SMALL:
                 assert nrows >= 16 or row0 > 0
+        else:                              # tcgen05 (opt-in): stacked rows in 128-row blocks
+            assert kind == 2 and flags & (tp.TP_DECODE_TCGEN05 | tp.TP_DECODE_ALL_TCGEN05)
+            assert 1 <= nrows <= 128
+            if flags & tp.TP_DECODE_ALL_TCGEN05:
+                assert row0 > 0 or nrows >= 17
+            else:
+                assert nt >= 32 and (row0 > 0 or nrows >= 64)
         tok = _expand(S["tiles"][toff:toff + nt])
         assert len(tok) > 0
         if row0 == 0:
@@ -296,7 +306,8 @@ def check_schedule(f, ids, model, script, leaves_sid, flags=0):
 
 
 @pytest.mark.parametrize("seed", range(6))
-@pytest.mark.parametrize("flags", [0, tp.TP_DECODE_NO_SHARE, tp.TP_DECODE_CUDA_CORE_SMALL])
+@pytest.mark.parametrize("flags", [0, tp.TP_DECODE_NO_SHARE, tp.TP_DECODE_CUDA_CORE_SMALL, tp.TP_DECODE_TCGEN05,
+                                   tp.TP_DECODE_ALL_TCGEN05])
 def test_schedule_covers_every_path_token_once(seed, flags):
     s = workloads.random_tree(seed=seed, n_prompts=3, max_depth=5, prompt_range=(1, 300), seg_range=(1, 150),
                               heads=workloads.Heads(8, 2, 64))
