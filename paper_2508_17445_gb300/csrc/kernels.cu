@@ -1500,30 +1500,64 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
     if (blockIdx.x == 0 && threadIdx.x < 3) a.counters[threadIdx.x] = 0;  // decode is done: re-arm its counters
     if (warp_global >= a.n * a.hq) return;
     const int i = warp_global / a.hq, qh = warp_global % a.hq;
-    const int beg = a.merge_off[i], end = a.merge_off[i + 1];
-    float M = -INFINITY;
-    for (int k = beg + lane; k < end; k += 32) M = fmaxf(M, a.part_lse[(int64_t)a.merge_slot[k] * a.hq + qh]);
-#pragma unroll
-    for (int off = 16; off; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    const int beg = a.merge_off[i], ns = a.merge_off[i + 1] - beg;
     float acc[DPL];
 #pragma unroll
     for (int d = 0; d < DPL; ++d) acc[d] = 0.f;
-    float L = 0.f;
-    for (int k = beg; k < end; ++k) {
-        const int64_t slot = a.merge_slot[k];
-        const float w = fast_exp2(a.part_lse[slot * a.hq + qh] - M);
-        L += w;
-        const float* src = a.part_o + (slot * a.hq + qh) * HD + lane * DPL;
-        if constexpr (DPL == 4) {
-            const float4 x = *reinterpret_cast<const float4*>(src);
-            acc[0] += w * x.x;
-            acc[1] += w * x.y;
-            acc[2] += w * x.z;
-            acc[3] += w * x.w;
-        } else {
-            const float2 x = *reinterpret_cast<const float2*>(src);
-            acc[0] += w * x.x;
-            acc[1] += w * x.y;
+    float M = -INFINITY, L = 0.f;
+    // slots in chunks of 32: lane k fetches slot k's index and LSE, then the
+    // warp folds the chunk's partial rows, four loads in flight per lane
+    for (int c0 = 0; c0 < ns; c0 += 32) {
+        const int k = c0 + lane;
+        int slot = 0;
+        float lse = -INFINITY;
+        if (k < ns) {
+            slot = a.merge_slot[beg + k];
+            lse = a.part_lse[(int64_t)slot * a.hq + qh];
+        }
+        float cm = lse;
+#pragma unroll
+        for (int off = 16; off; off >>= 1) cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, off));
+        const float m_new = fmaxf(M, cm);
+        const float keep = (M == -INFINITY) ? 0.f : fast_exp2(M - m_new);
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) acc[d] *= keep;
+        L *= keep;
+        M = m_new;
+        const float w = (k < ns) ? fast_exp2(lse - M) : 0.f;
+        float ws = w;
+#pragma unroll
+        for (int off = 16; off; off >>= 1) ws += __shfl_xor_sync(0xffffffffu, ws, off);
+        L += ws;
+        const int cnt = min(32, ns - c0);
+        int j = 0;
+        for (; j + 4 <= cnt; j += 4) {
+            float wj[4];
+            float x[4][DPL];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int64_t sl = __shfl_sync(0xffffffffu, slot, j + u);
+                wj[u] = __shfl_sync(0xffffffffu, w, j + u);
+                const float* src = a.part_o + (sl * a.hq + qh) * HD + lane * DPL;
+                if constexpr (DPL == 4) {
+                    const float4 v = *reinterpret_cast<const float4*>(src);
+                    x[u][0] = v.x, x[u][1] = v.y, x[u][2] = v.z, x[u][3] = v.w;
+                } else {
+                    const float2 v = *reinterpret_cast<const float2*>(src);
+                    x[u][0] = v.x, x[u][1] = v.y;
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int d = 0; d < DPL; ++d) acc[d] += wj[u] * x[u][d];
+        }
+        for (; j < cnt; ++j) {
+            const int64_t sl = __shfl_sync(0xffffffffu, slot, j);
+            const float wj = __shfl_sync(0xffffffffu, w, j);
+            const float* src = a.part_o + (sl * a.hq + qh) * HD + lane * DPL;
+#pragma unroll
+            for (int d = 0; d < DPL; ++d) acc[d] += wj * src[d];
         }
     }
     const float inv = 1.f / L;
