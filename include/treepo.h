@@ -192,6 +192,20 @@ tp_status tp_decode_ex(tp_tree* tree, const tp_node* leaves, int32_t n, const vo
 tp_status tp_decode_noalloc(tp_tree* tree, const tp_node* leaves, int32_t n, const void* Q, void* O,
                             float* LSE, uint32_t flags);
 
+/*
+ * Decode-loop append: one token to each of n distinct live leaves (the step
+ * of token-level decoding inside a segment, Sec. 2.2). Row i of K and V
+ * (device bf16 [n][num_kv_heads][head_dim], 16-byte aligned) becomes the
+ * next token of nodes[i] (host array). Equivalent to n calls of
+ * tp_append_segment with one token each, in one kernel launch. A decode of
+ * the same leaf list after appends that stayed inside the leaves' last
+ * blocks reuses its cached schedule (only the leaves' last-block token
+ * counts are rewritten on the device). n == 0 is a no-op. Errors:
+ * TP_ERR_BAD_NODE, TP_ERR_FROZEN, TP_ERR_OOM (nothing is appended),
+ * TP_ERR_INVALID_ARG (also for a node listed twice).
+ */
+tp_status tp_append_tokens(tp_tree* tree, const tp_node* nodes, int32_t n, const void* K, const void* V);
+
 /* Wait for the tree's stream; TP_ERR_DEVICE if a kernel gave up a bounded
  * wait since the last tp_sync (the flag is then cleared), TP_ERR_CUDA on a
  * CUDA error. */
@@ -233,6 +247,191 @@ typedef struct {
 } tp_kernel_times;
 tp_status tp_profile_start(tp_tree* tree);
 tp_status tp_profile_stop(tp_tree* tree, tp_kernel_times* out);
+
+/* ---- tree sampling (Sec. 2.2, Algorithm 1) ------------------------------ */
+
+/*
+ * Branching budget split (Sec. 2.2 budget transfer; Sec. 4.6 probability-
+ * based assignment): out[i] >= 1 branches for each of n active paths,
+ * summing to budget (>= n). Policies:
+ *   TP_BRANCH_EVEN       out[i] = budget / n, plus one for the first
+ *                        budget % n paths (logp unused, may be NULL);
+ *   TP_BRANCH_LOGP_HIGH  the budget - n branches beyond the first one per
+ *   TP_BRANCH_LOGP_LOW   path are split by softmax(+-logp / temperature)
+ *                        (HIGH favours paths whose last segment had the
+ *                        higher log-probability, LOW the lower), rounded by
+ *                        largest remainder, ties to the lower index.
+ * logp: host double [n] (finite); out: host int32 [n]. Computed in double
+ * precision in index order. Errors: TP_ERR_INVALID_ARG (budget < n,
+ * temperature <= 0, non-finite logp, unknown policy).
+ */
+#define TP_BRANCH_EVEN 0
+#define TP_BRANCH_LOGP_HIGH 1
+#define TP_BRANCH_LOGP_LOW 2
+tp_status tp_branch_assign(const double* logp, int32_t n, int32_t budget, int32_t policy, double temperature,
+                           int32_t* out);
+
+/*
+ * Rollout parameters. The language model is replaced by a synthetic stand-
+ * in whose every draw is SplitMix64 (Steele et al. 2014) element
+ *   mix(seed + (ctr + 1) * 0x9E3779B97F4A7C15),
+ *   ctr = tag << 60 | a << 32 | b << 12 | c   (a < 2^28, b < 2^20, c < 2^12),
+ * read as u = (x >> 11) * 2^-53 in [0, 1) for decisions, or as four bf16
+ * values (16 bits each, low bits first: sign bit 15, exponent 125 + bits
+ * 7..8, mantissa bits 0..6; values in +-[0.25, 4)) for activations:
+ *   K, V, Q of token b of node a: tags 1, 2, 3, c = word of the row
+ *       ([heads][head_dim] row-major, 4 values per word);
+ *   token b of segment node a is EOS if u(4, a, b, 0) < p_eos (the segment
+ *       ends there; else it has seg_tokens tokens); its log-probability is
+ *       kappa * ln(1 - u(5, a, b, 0)) with kappa = 2 u(6, a, 0, 0); the
+ *       segment's logp is the mean over its tokens;
+ *   the segment is "boxed" if u(6, a, 1, 0) < p_boxed, fails the
+ *       repetition check if u(6, a, 2, 0) < p_fail; a boxed trajectory
+ *       earns reward 1 if u(6, a, 3, 0) < p_correct, else 0;
+ *   query q: b0 = 2 + floor(7 u(7, q, 0, 0)) when init_branches == 0; its
+ *       k-th fallback picks candidate floor(m u(7, q, 1, k)) of its m live
+ *       candidates and boundary floor(J u(7, q, 2, k)) of that candidate's
+ *       J segments.
+ * Algorithm 1 with these readings:
+ *   - each query is a root holding prompt_tokens[q] tokens (depth 0), forked
+ *     into min(b0, w) paths; each queued path generates one segment per
+ *     loop pass as a new node (depth = parent's + 1);
+ *   - a segment that fails is an output and is pruned at once; one that
+ *     ends in EOS, is boxed or reaches max_depth finishes its trajectory
+ *     (an output; a candidate for fallback if EOS or boxed); every other
+ *     path continues;
+ *   - branching: the continuing paths of query q at depth j are forked to
+ *     min(b0 * arity^j, w - outputs_q) paths (never fewer than one each),
+ *     split by `policy`; queries in ascending order, paths in queue order;
+ *   - fallback (if enabled): after branching, a query with no path and
+ *     fewer than w outputs forks one new path from the chosen boundary
+ *     node of a live candidate; candidates stay alive (their KV kept) until
+ *     their query is done, otherwise finished paths are pruned at once;
+ *   - a query with no path after fallback is done: its candidates are pruned.
+ * With decode != 0 (device pool needed), every generated token is appended
+ * with tp_append_tokens and the paths still generating decode (tp_decode_ex
+ * with decode_flags); with decode == 0 each segment is appended whole.
+ */
+typedef struct {
+    int32_t n_queries;
+    const int32_t* prompt_tokens; /* host [n_queries], each in [1, 2^20] */
+    int32_t width;                /* w >= 1: trajectories per query      */
+    int32_t max_depth;            /* d >= 1: segments per trajectory     */
+    int32_t seg_tokens;           /* l >= 1: tokens per segment          */
+    int32_t arity;                /* N >= 1                              */
+    int32_t init_branches;        /* b0 >= 1, or 0: b0 drawn in [2, 8]   */
+    int32_t policy;               /* TP_BRANCH_*                         */
+    int32_t fallback;             /* nonzero: depth-first-search fallback */
+    int32_t decode;               /* nonzero: decode after every token   */
+    uint32_t decode_flags;        /* tp_decode_ex flags                  */
+    int32_t reserved;
+    double temperature;           /* > 0 for the log-prob policies       */
+    double p_eos, p_boxed, p_fail, p_correct;
+    uint64_t seed;
+} tp_rollout_params;
+
+/* Segment status bits (event TP_EV_SEGMENT). */
+#define TP_SEG_EOS 1
+#define TP_SEG_BOXED 2
+#define TP_SEG_FAILED 4
+#define TP_SEG_MAX_DEPTH 8
+
+/* Events: int64 records of 8 words {kind, query, node, a, b, c, d, 0}.
+ *   TP_EV_ROOT      node = root, a = prompt tokens, b = b0
+ *   TP_EV_FORK      node = parent, a = first child (children are
+ *                   consecutive ids), b = k
+ *   TP_EV_SEGMENT   node, a = depth, b = tokens, c = TP_SEG_* bits,
+ *                   d = bits of the double segment logp
+ *   TP_EV_OUTPUT    node = leaf, a = depth, b = fallback candidate, c = reward
+ *   TP_EV_PRUNE     node = leaf
+ *   TP_EV_FALLBACK  node = candidate leaf, a = boundary node, b = its depth
+ *   TP_EV_DONE      node = -1, a = outputs of the query */
+#define TP_EV_ROOT 1
+#define TP_EV_FORK 2
+#define TP_EV_SEGMENT 3
+#define TP_EV_OUTPUT 4
+#define TP_EV_PRUNE 5
+#define TP_EV_FALLBACK 6
+#define TP_EV_DONE 7
+
+typedef struct {
+    int64_t iterations;    /* loop passes (Inference calls)          */
+    int64_t segments;      /* generated segments                     */
+    int64_t tokens;        /* generated tokens                       */
+    int64_t prompt_tokens; /* prompt tokens appended                 */
+    int64_t outputs;       /* trajectories in O                      */
+    int64_t fallbacks;
+    int64_t decode_calls;
+    int64_t decode_rows;   /* leaf queries over all decode calls     */
+    int64_t events;        /* events produced (may exceed the cap)   */
+    int64_t peak_blocks;   /* most pool blocks in use at once        */
+    int64_t nodes;         /* nodes created                          */
+} tp_rollout_stats;
+
+/* Optional copy-out of one decode call of a rollout (for checking it): the
+ * call with index `call` (0-based over the rollout) copies its first
+ * min(rows, cap) rows of O (device bf16 [cap][num_q_heads][head_dim]) and
+ * LSE (device fp32 [cap][num_q_heads]); rows (host int32 [cap][2]) gets
+ * each row's (leaf node, token index inside the leaf), *n_rows the count. */
+typedef struct {
+    int64_t call;
+    int32_t cap;
+    int32_t reserved;
+    void* o;
+    float* lse;
+    int32_t* rows;
+    int32_t* n_rows;
+} tp_rollout_probe;
+
+/*
+ * Run Algorithm 1 for p->n_queries new prompts in `tree` (roots are added
+ * to whatever the tree holds). events: host int64 [cap_events][8] or NULL;
+ * stats->events tells how many were produced. probe, stats: optional.
+ * Returns when the rollout is done; device work is enqueued on the tree's
+ * stream. On error the rollout stops where it failed (the tree keeps what
+ * was built). Errors: TP_ERR_INVALID_ARG, TP_ERR_OOM (pool exhausted),
+ * and those of the calls above.
+ */
+tp_status tp_rollout(tp_tree* tree, const tp_rollout_params* params, int64_t* events, int64_t cap_events,
+                     const tp_rollout_probe* probe, tp_rollout_stats* stats);
+
+/*
+ * Stand-in activations, as the rollout draws them: K, V ([n][num_kv_heads]
+ * [head_dim]) and Q ([n][num_q_heads][head_dim]) bf16 rows of tokens
+ * pos0 .. pos0 + n - 1 of node key `node` (device pointers, 8-byte aligned,
+ * any may be NULL). The paper has no counterpart; it exposes the synthetic
+ * inputs so they can be checked. node < 2^28, pos0 + n <= 2^20.
+ */
+tp_status tp_synth_tokens(tp_tree* tree, uint64_t seed, tp_node node, int32_t pos0, int32_t n_tokens, void* K,
+                          void* V, void* Q);
+
+/* ---- tree advantage (Sec. 2.3, Eq. tree_ae) ----------------------------- */
+
+/*
+ * Advantage of each trajectory from the sub-groups of the tree. Trajectory
+ * i ends at node leaf[i] with reward[i]; its sub-groups are the strict
+ * ancestors x of leaf[i] (depth 0 = the query's root, through the leaf's
+ * parent), G_x = the trajectories below x. Then
+ *   A_i   = (1 / |J_i|) sum_{x in J_i} (R_i - mean_{G_x} R)   (mean pooling)
+ *   adv_i = A_i / std(A)                       (global normalisation)
+ * where std is the population standard deviation over every accepted
+ * trajectory of the call. A trajectory is rejected (adv 0, left out of the
+ * std) when all rewards of its query (root) are equal (std(R) = 0) or its
+ * leaf is a root; adv is 0 everywhere when std(A) = 0.
+ * parent: device int32 [n_nodes] (-1 for roots; parent ids need not be
+ * smaller than their children's), leaf: device int32 [n_out], reward:
+ * device fp32 [n_out] (finite), adv: device fp32 [n_out]. stats: device
+ * double [4] or NULL: accepted trajectories, mean(A), std(A), and 1 if the
+ * parent table was malformed (an id out of range or a cycle; the affected
+ * trajectories are rejected). workspace: device, 8-byte aligned, at least
+ * tp_advantage_workspace_bytes(n_nodes, n_out) bytes. Fp64 accumulation,
+ * one CTA, asynchronous on cuda_stream. Errors (tp_last_error(NULL)):
+ * TP_ERR_INVALID_ARG, TP_ERR_CUDA.
+ */
+int64_t tp_advantage_workspace_bytes(int32_t n_nodes, int32_t n_out);
+tp_status tp_tree_advantage(const int32_t* parent, int32_t n_nodes, const int32_t* leaf, const float* reward,
+                            int32_t n_out, float* adv, double* stats, void* workspace, int64_t workspace_bytes,
+                            void* cuda_stream);
 
 /* ---- inspection (tests and tools) ------------------------------------ */
 

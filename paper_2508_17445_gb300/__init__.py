@@ -23,7 +23,10 @@ __all__ = [
     "tp_set_stream", "tp_add_root", "tp_append_segment", "tp_fork", "tp_prune", "tp_decode", "tp_decode_ex",
     "tp_sync", "tp_last_error", "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop",
     "tp_debug_path", "tp_debug_gather",
-    "tp_debug_schedule", "tp_decode_noalloc", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE", "TP_DECODE_TCGEN05", "TP_DECODE_ALL_TCGEN05",
+    "tp_debug_schedule", "tp_decode_noalloc", "tp_append_tokens", "tp_synth_tokens", "tp_branch_assign",
+    "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "TpRolloutParams", "TpRolloutStats",
+    "TpRolloutProbe", "rollout_params", "TP_BRANCH_EVEN", "TP_BRANCH_LOGP_HIGH", "TP_BRANCH_LOGP_LOW",
+    "EVENT_NAMES", "TP_SEG_EOS", "TP_SEG_BOXED", "TP_SEG_FAILED", "TP_SEG_MAX_DEPTH", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE", "TP_DECODE_TCGEN05", "TP_DECODE_ALL_TCGEN05",
     "EXPORTED_SYMBOLS",
 ]
 
@@ -37,6 +40,12 @@ TP_DECODE_NO_CACHE = 4
 TP_DECODE_TCGEN05 = 8
 TP_DECODE_ALL_TCGEN05 = 16
 
+TP_BRANCH_EVEN = 0
+TP_BRANCH_LOGP_HIGH = 1
+TP_BRANCH_LOGP_LOW = 2
+TP_SEG_EOS, TP_SEG_BOXED, TP_SEG_FAILED, TP_SEG_MAX_DEPTH = 1, 2, 4, 8
+EVENT_NAMES = {1: "root", 2: "fork", 3: "segment", 4: "output", 5: "prune", 6: "fallback", 7: "done"}
+
 STATUS_NAMES = {0: "OK", -1: "INVALID_ARG", -2: "OOM", -3: "BAD_NODE", -4: "FROZEN", -5: "NOT_LEAF",
                 -6: "EMPTY_PATH", -7: "CUDA", -8: "DEVICE"}
 
@@ -44,7 +53,8 @@ EXPORTED_SYMBOLS = (
     "tp_pool_bytes", "tp_tree_create", "tp_tree_destroy", "tp_set_stream", "tp_add_root",
     "tp_append_segment", "tp_fork", "tp_prune", "tp_decode", "tp_decode_ex", "tp_sync", "tp_last_error",
     "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop", "tp_debug_path",
-    "tp_debug_gather", "tp_debug_schedule", "tp_decode_noalloc",
+    "tp_debug_gather", "tp_debug_schedule", "tp_decode_noalloc", "tp_append_tokens", "tp_synth_tokens",
+    "tp_branch_assign", "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage",
 )
 
 
@@ -71,6 +81,27 @@ class TpKernelTimes(ctypes.Structure):
 
 
 KERNEL_KINDS = ("decode", "merge", "append", "gather")
+
+
+class TpRolloutParams(ctypes.Structure):
+    _fields_ = [("n_queries", ctypes.c_int32), ("prompt_tokens", ctypes.c_void_p), ("width", ctypes.c_int32),
+                ("max_depth", ctypes.c_int32), ("seg_tokens", ctypes.c_int32), ("arity", ctypes.c_int32),
+                ("init_branches", ctypes.c_int32), ("policy", ctypes.c_int32), ("fallback", ctypes.c_int32),
+                ("decode", ctypes.c_int32), ("decode_flags", ctypes.c_uint32), ("reserved", ctypes.c_int32),
+                ("temperature", ctypes.c_double), ("p_eos", ctypes.c_double), ("p_boxed", ctypes.c_double),
+                ("p_fail", ctypes.c_double), ("p_correct", ctypes.c_double), ("seed", ctypes.c_uint64)]
+
+
+class TpRolloutStats(ctypes.Structure):
+    _fields_ = [(f, ctypes.c_int64) for f in ("iterations", "segments", "tokens", "prompt_tokens", "outputs",
+                                               "fallbacks", "decode_calls", "decode_rows", "events",
+                                               "peak_blocks", "nodes")]
+
+
+class TpRolloutProbe(ctypes.Structure):
+    _fields_ = [("call", ctypes.c_int64), ("cap", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("o", ctypes.c_void_p), ("lse", ctypes.c_void_p), ("rows", ctypes.c_void_p),
+                ("n_rows", ctypes.c_void_p)]
 
 
 class TpStats(ctypes.Structure):
@@ -113,6 +144,12 @@ def load_library() -> ctypes.CDLL:
         "tp_debug_path": (I32, [P, I32, P, I64, P]),
         "tp_debug_gather": (I32, [P, I32, P, P, I64, P]),
         "tp_debug_schedule": (I32, [P, P, I32, U32, P, I64, P]),
+        "tp_append_tokens": (I32, [P, P, I32, P, P]),
+        "tp_synth_tokens": (I32, [P, ctypes.c_uint64, I32, I32, I32, P, P, P]),
+        "tp_branch_assign": (I32, [P, I32, I32, I32, ctypes.c_double, P]),
+        "tp_rollout": (I32, [P, P, P, I64, P, P]),
+        "tp_advantage_workspace_bytes": (I64, [I32, I32]),
+        "tp_tree_advantage": (I32, [P, I32, P, P, I32, P, P, P, I64, P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -269,6 +306,68 @@ def tp_debug_schedule(h, leaves: Sequence[int], flags: int = 0) -> Dict[str, np.
             "n_slots": n_slots, "group": g, "n_tensor_units": n_tensor, "n_tc_units": n_tc, "words": w}
 
 
+def tp_append_tokens(h, nodes: Sequence[int], K=None, V=None) -> None:
+    """One token per node; K, V: device bf16 [n][Hkv][hd] (None on a metadata-only tree)."""
+    arr = _node_array(nodes)
+    _check(h, load_library().tp_append_tokens(h, arr.ctypes.data if len(arr) else None, len(arr), _ptr(K), _ptr(V)))
+
+
+def tp_synth_tokens(h, seed: int, node: int, pos0: int, n_tokens: int, K=None, V=None, Q=None) -> None:
+    _check(h, load_library().tp_synth_tokens(h, seed, node, pos0, n_tokens, _ptr(K), _ptr(V), _ptr(Q)))
+
+
+def tp_branch_assign(logp: Optional[Sequence[float]], n: int, budget: int, policy: int,
+                     temperature: float = 1.0) -> List[int]:
+    lp = None if logp is None else np.ascontiguousarray(np.asarray(logp, dtype=np.float64))
+    out = np.zeros(max(n, 1), dtype=np.int32)
+    st = load_library().tp_branch_assign(None if lp is None else lp.ctypes.data, n, budget, policy,
+                                         float(temperature), out.ctypes.data)
+    if st != 0:
+        raise TreepoError(st, "tp_branch_assign rejected its arguments")
+    return [int(x) for x in out[:n]]
+
+
+def rollout_params(prompt_tokens: Sequence[int], **kw) -> TpRolloutParams:
+    """Parameters with defaults: w=16, d=14, l=512, binary, b0=2, even split,
+    fallback on, no decode, T=2.0; ``prompt_tokens`` is kept alive on the
+    returned object."""
+    arr = np.ascontiguousarray(np.asarray(prompt_tokens, dtype=np.int32))
+    d = dict(width=16, max_depth=14, seg_tokens=512, arity=2, init_branches=2, policy=TP_BRANCH_EVEN, fallback=1,
+             decode=0, decode_flags=0, temperature=2.0, p_eos=0.0, p_boxed=0.0, p_fail=0.0, p_correct=0.5, seed=0)
+    d.update(kw)
+    p = TpRolloutParams(n_queries=len(arr), prompt_tokens=arr.ctypes.data, reserved=0, **d)
+    p._prompts = arr
+    return p
+
+
+def tp_rollout(h, params: TpRolloutParams, cap_events: int = 1 << 20, probe: Optional[TpRolloutProbe] = None):
+    """Run Algorithm 1; returns (events int64 [n][8], stats dict)."""
+    ev = np.zeros((max(cap_events, 1), 8), dtype=np.int64)
+    st = TpRolloutStats()
+    _check(h, load_library().tp_rollout(h, ctypes.byref(params), ev.ctypes.data, cap_events,
+                                        ctypes.byref(probe) if probe is not None else None, ctypes.byref(st)))
+    stats = {f: int(getattr(st, f)) for f, _ in TpRolloutStats._fields_}
+    if stats["events"] > cap_events:
+        raise TreepoError(-1, f"{stats['events']} events exceed cap_events={cap_events}")
+    return ev[: stats["events"]].copy(), stats
+
+
+def tp_advantage_workspace_bytes(n_nodes: int, n_out: int) -> int:
+    return int(load_library().tp_advantage_workspace_bytes(n_nodes, n_out))
+
+
+def tp_tree_advantage(parent, leaf, reward, adv, stats=None, workspace=None, stream: int = 0) -> None:
+    """parent int32 [n_nodes], leaf int32 [n_out], reward / adv float32 [n_out], stats float64 [4] (device tensors)."""
+    ws_bytes = tp_advantage_workspace_bytes(int(parent.shape[0]), int(leaf.shape[0]))
+    if workspace is None:
+        import torch
+        workspace = torch.empty(max(ws_bytes, 8), dtype=torch.uint8, device=parent.device)
+    st = load_library().tp_tree_advantage(_ptr(parent), int(parent.shape[0]), _ptr(leaf), _ptr(reward),
+                                          int(leaf.shape[0]), _ptr(adv), _ptr(stats), _ptr(workspace),
+                                          int(workspace.numel()), stream)
+    _check(None, st)
+
+
 # ------------------------------------------------------------------ owner --
 class Forest:
     """A tp_tree plus the pool arena it owns.
@@ -334,6 +433,12 @@ class Forest:
             O, LSE = out
         tp_decode_ex(self.handle, leaves, Q, O, LSE, flags)
         return O, LSE
+
+    def append_tokens(self, nodes: Sequence[int], K=None, V=None) -> None:
+        tp_append_tokens(self.handle, nodes, K, V)
+
+    def rollout(self, params: TpRolloutParams, cap_events: int = 1 << 20, probe=None):
+        return tp_rollout(self.handle, params, cap_events, probe)
 
     def sync(self) -> None:
         tp_sync(self.handle)

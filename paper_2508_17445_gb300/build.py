@@ -18,7 +18,7 @@ ROOT = os.path.dirname(HERE)
 LIB = os.path.join(HERE, "libtreepo.so")
 BUILD_DIR = os.path.join(HERE, "_build")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["kernels.cu", "forest.cpp", "capi.cpp"]
+SOURCES = ["kernels.cu", "forest.cpp", "capi.cpp", "rollout.cpp"]
 
 
 def _nvcc() -> str:
@@ -49,7 +49,9 @@ def build(force: bool = False, verbose: bool = False) -> str:
         if src.endswith(".cu"):
             cmd[1:1] = [*ARCH, "-lineinfo", "-Xptxas", "-v" if verbose else "-O3"]
         else:
-            cmd[1:1] = ["-x", "c++"]
+            # no fused multiply-add contraction: host decisions that compare
+            # doubles (branch splits) must round the same on every machine
+            cmd[1:1] = ["-x", "c++", "-Xcompiler", "-ffp-contract=off"]
         res = subprocess.run(cmd, capture_output=True, text=True)
         if res.returncode != 0:
             raise RuntimeError(f"compiling {src} failed:\n{' '.join(cmd)}\n{res.stdout}\n{res.stderr}")

@@ -9,43 +9,33 @@
 
 using tp::fail;
 
-namespace {
-
-thread_local std::string g_create_err;
-
-bool aligned(const void* p, uintptr_t a) { return ((uintptr_t)p % a) == 0; }
+namespace tp {
 
 tp_status cuda_fail(tp_tree* t, cudaError_t e, const char* what) {
     return fail(t, TP_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
 }
 
-// Grow a device buffer; waits for the stream so no queued kernel still reads it.
-template <typename T>
-tp_status ensure_device(tp_tree* t, T*& ptr, int64_t& cap, int64_t need, const char* what) {
-    if (need <= cap) return TP_OK;
-    int64_t want = std::max<int64_t>(need, cap + cap / 2);
-    if (ptr) {
+tp_status ensure_device_bytes(tp_tree* t, void** ptr, int64_t* cap, int64_t need, const char* what) {
+    if (need <= *cap) return TP_OK;
+    int64_t want = std::max<int64_t>(need, *cap + *cap / 2);
+    if (*ptr) {
         cudaStreamSynchronize(t->stream);
-        cudaFree(ptr);
-        ptr = nullptr;
-        cap = 0;
+        cudaFree(*ptr);
+        *ptr = nullptr;
+        *cap = 0;
     }
-    cudaError_t e = cudaMalloc((void**)&ptr, (size_t)want * sizeof(T));
+    cudaError_t e = cudaMalloc(ptr, (size_t)want);
     if (e != cudaSuccess) {
-        ptr = nullptr;
+        *ptr = nullptr;
         cudaGetLastError();
         return fail(t, e == cudaErrorMemoryAllocation ? TP_ERR_OOM : TP_ERR_CUDA,
                     std::string(what) + ": " + cudaGetErrorString(e));
     }
-    cap = want;
+    *cap = want;
     return TP_OK;
 }
 
-// Copy a schedule to the device through a double-buffered pinned staging area.
-tp_status upload_schedule(tp_tree* t, const tp::Schedule& s) {
-    const int64_t words = (int64_t)s.words.size();
-    tp_status st = ensure_device(t, t->d_sched, t->d_sched_cap, words, "schedule buffer");
-    if (st != TP_OK) return st;
+tp_status stage_upload(tp_tree* t, int32_t* dst, const int32_t* src, int64_t words) {
     const int k = t->pinned_next;
     t->pinned_next ^= 1;
     if (t->h_pinned_ev[k] == nullptr) {
@@ -63,11 +53,54 @@ tp_status upload_schedule(tp_tree* t, const tp::Schedule& s) {
         if (e != cudaSuccess) return cuda_fail(t, e, "cudaHostAlloc");
         t->h_pinned_cap[k] = want;
     }
-    std::memcpy(t->h_pinned[k], s.words.data(), (size_t)words * 4);
-    e = cudaMemcpyAsync(t->d_sched, t->h_pinned[k], (size_t)words * 4, cudaMemcpyHostToDevice, t->stream);
-    if (e != cudaSuccess) return cuda_fail(t, e, "schedule upload");
+    std::memcpy(t->h_pinned[k], src, (size_t)words * 4);
+    e = cudaMemcpyAsync(dst, t->h_pinned[k], (size_t)words * 4, cudaMemcpyHostToDevice, t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "host-to-device upload");
     e = cudaEventRecord(t->h_pinned_ev[k], t->stream);
     if (e != cudaSuccess) return cuda_fail(t, e, "cudaEventRecord");
+    return TP_OK;
+}
+
+}  // namespace tp
+
+namespace {
+
+using tp::cuda_fail;
+using tp::stage_upload;
+
+thread_local std::string g_create_err;
+
+bool aligned(const void* p, uintptr_t a) { return ((uintptr_t)p % a) == 0; }
+
+// Grow a typed device buffer (counted in elements).
+template <typename T>
+tp_status ensure_device(tp_tree* t, T*& ptr, int64_t& cap, int64_t need, const char* what) {
+    void* p = ptr;
+    int64_t bytes = cap * (int64_t)sizeof(T);
+    tp_status st = tp::ensure_device_bytes(t, &p, &bytes, need * (int64_t)sizeof(T), what);
+    ptr = (T*)p;
+    cap = bytes / (int64_t)sizeof(T);
+    return st;
+}
+
+tp_status upload_schedule(tp_tree* t, const tp::Schedule& s) {
+    const int64_t words = (int64_t)s.words.size();
+    tp_status st = ensure_device(t, t->d_sched, t->d_sched_cap, words, "schedule buffer");
+    if (st != TP_OK) return st;
+    return stage_upload(t, t->d_sched, s.words.data(), words);
+}
+
+// Bring the cached device schedule up to date after appends that stayed
+// inside the listed leaves' last blocks: only their last-tile words change.
+tp_status patch_cached_schedule(tp_tree* t) {
+    const int32_t n = tp::patch_schedule(t, t->sched, t->patch_words);
+    if (n == 0) return TP_OK;
+    tp_status st = ensure_device(t, t->d_patch, t->d_patch_cap, 2 * (int64_t)n, "schedule patch buffer");
+    if (st != TP_OK) return st;
+    st = stage_upload(t, t->d_patch, t->patch_words.data(), 2 * (int64_t)n);
+    if (st != TP_OK) return st;
+    cudaError_t e = tp::launch_patch(t->d_sched, t->d_patch, n, t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "schedule patch kernel");
     return TP_OK;
 }
 
@@ -150,6 +183,8 @@ tp_status tp_tree_destroy(tp_tree* t) {
     if (t->d_sched) cudaFree(t->d_sched);
     if (t->d_part) cudaFree(t->d_part);
     if (t->d_gather_tiles) cudaFree(t->d_gather_tiles);
+    if (t->d_patch) cudaFree(t->d_patch);
+    if (t->d_tok_slots) cudaFree(t->d_tok_slots);
     for (cudaEvent_t e : t->ev_pool) cudaEventDestroy(e);
     if (t->ev_fork) cudaEventDestroy(t->ev_fork);
     if (t->ev_join) cudaEventDestroy(t->ev_join);
@@ -175,6 +210,7 @@ tp_status tp_add_root(tp_tree* t, tp_node* out) {
     *out = (tp_node)t->nodes.size() - 1;
     ++t->live_nodes;
     ++t->version;
+    ++t->struct_version;
     return TP_OK;
 }
 
@@ -234,6 +270,144 @@ tp_status tp_append_segment(tp_tree* t, tp_node node, int32_t n_tokens, const vo
     }
     nd.n_tokens += n_tokens;
     ++t->version;
+    if (need > 0) ++t->struct_version;
+    return TP_OK;
+}
+
+tp_status tp_append_tokens(tp_tree* t, const tp_node* nodes, int32_t n, const void* K, const void* V) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    if (n < 0) return fail(t, TP_ERR_INVALID_ARG, "n < 0");
+    if (n == 0) return TP_OK;
+    if (!nodes) return fail(t, TP_ERR_INVALID_ARG, "nodes is NULL");
+    if (t->cfg.pool) {
+        if (!K || !V || !aligned(K, 16) || !aligned(V, 16))
+            return fail(t, TP_ERR_INVALID_ARG, "K and V must be non-NULL 16-byte aligned device pointers");
+    } else if (K || V) {
+        return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree: K and V must be NULL");
+    }
+    tp::SchedScratch& X = t->scratch;
+    if (X.mark.size() < t->nodes.size()) {
+        X.mark.resize(t->nodes.size(), 0);
+        X.local.resize(t->nodes.size(), 0);
+    }
+    if (++X.epoch == 0) {
+        std::fill(X.mark.begin(), X.mark.end(), 0u);
+        X.epoch = 1;
+    }
+    const int32_t bt = t->cfg.block_tokens;
+    int64_t need = 0;
+    for (int32_t i = 0; i < n; ++i) {
+        tp_status st = tp::check_live(t, nodes[i], false);
+        if (st != TP_OK) return st;
+        const tp::Node& nd = t->nodes[(size_t)nodes[i]];
+        if (nd.state != 0) return fail(t, TP_ERR_FROZEN, "node " + std::to_string(nodes[i]) + " has been forked");
+        if (X.mark[(size_t)nodes[i]] == X.epoch)
+            return fail(t, TP_ERR_INVALID_ARG, "node " + std::to_string(nodes[i]) + " is listed twice");
+        if (nd.n_tokens >= INT32_MAX / 2) return fail(t, TP_ERR_INVALID_ARG, "node too long");
+        X.mark[(size_t)nodes[i]] = X.epoch;
+        need += nd.n_tokens % bt == 0;
+    }
+    if (need > t->pool.free_count())
+        return fail(t, TP_ERR_OOM, "pool exhausted: need " + std::to_string(need) + " blocks, " +
+                                       std::to_string(t->pool.free_count()) + " free");
+    std::vector<int32_t>& slots = t->tok_slots;
+    slots.resize((size_t)n);
+    for (int32_t i = 0; i < n; ++i) {
+        tp::Node& nd = t->nodes[(size_t)nodes[i]];
+        if (nd.n_tokens % bt == 0) t->pool.alloc(1, nd.blocks);  // cannot fail: counted above
+        slots[(size_t)i] = nd.blocks[(size_t)(nd.n_tokens / bt)] * bt + nd.n_tokens % bt;
+    }
+    if (t->cfg.pool) {
+        tp_status st = ensure_device(t, t->d_tok_slots, t->d_tok_slots_cap, n, "token slot buffer");
+        if (st == TP_OK) st = stage_upload(t, t->d_tok_slots, slots.data(), n);
+        cudaError_t e = cudaSuccess;
+        if (st == TP_OK) {
+            tp::AppendTokensArgs a;
+            a.k = K;
+            a.v = V;
+            a.slots = t->d_tok_slots;
+            a.pool = (uint8_t*)t->cfg.pool;
+            a.head_bytes = bt * t->cfg.head_dim * 2;
+            a.block_bytes = (int64_t)2 * t->cfg.num_kv_heads * a.head_bytes;
+            a.hkv = t->cfg.num_kv_heads;
+            a.n = n;
+            tp::LaunchTimer timer(t, tp::KK_APPEND);
+            e = tp::launch_append_tokens(t->cfg.head_dim, a, t->stream);
+            if (e != cudaSuccess) st = cuda_fail(t, e, "token append kernel");
+        }
+        if (st != TP_OK) {  // undo the block allocations
+            for (int32_t i = 0; i < n; ++i) {
+                tp::Node& nd = t->nodes[(size_t)nodes[i]];
+                if (nd.n_tokens % bt == 0) {
+                    t->pool.release({nd.blocks.back()});
+                    nd.blocks.pop_back();
+                }
+            }
+            return st;
+        }
+    }
+    for (int32_t i = 0; i < n; ++i) ++t->nodes[(size_t)nodes[i]].n_tokens;
+    ++t->version;
+    if (need > 0) ++t->struct_version;
+    return TP_OK;
+}
+
+tp_status tp_synth_tokens(tp_tree* t, uint64_t seed, tp_node node, int32_t pos0, int32_t n_tokens, void* K, void* V,
+                          void* Q) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    if (!t->cfg.pool) return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree launches no kernels");
+    if (node < 0 || node >= (1 << 28)) return fail(t, TP_ERR_INVALID_ARG, "node key must be in [0, 2^28)");
+    if (pos0 < 0 || n_tokens < 0 || (int64_t)pos0 + n_tokens > (1 << 20))
+        return fail(t, TP_ERR_INVALID_ARG, "token positions must lie in [0, 2^20)");
+    if ((K && !aligned(K, 8)) || (V && !aligned(V, 8)) || (Q && !aligned(Q, 8)))
+        return fail(t, TP_ERR_INVALID_ARG, "K, V and Q must be 8-byte aligned device pointers");
+    tp::SynthArgs a;
+    a.k = (uint16_t*)K;
+    a.v = (uint16_t*)V;
+    a.q = (uint16_t*)Q;
+    a.row_node = nullptr;
+    a.seed = seed;
+    a.rows = n_tokens;
+    a.kv_width = t->cfg.num_kv_heads * t->cfg.head_dim;
+    a.q_width = t->cfg.num_q_heads * t->cfg.head_dim;
+    a.node0 = node;
+    a.pos0 = pos0;
+    cudaError_t e = tp::launch_synth(a, t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "synth kernel");
+    return TP_OK;
+}
+
+int64_t tp_advantage_workspace_bytes(int32_t n_nodes, int32_t n_out) {
+    if (n_nodes < 0 || n_out < 0) return -1;
+    return tp::advantage_ws_bytes(n_nodes, n_out);
+}
+
+tp_status tp_tree_advantage(const int32_t* parent, int32_t n_nodes, const int32_t* leaf, const float* reward,
+                            int32_t n_out, float* adv, double* stats, void* workspace, int64_t workspace_bytes,
+                            void* cuda_stream) {
+    auto bad = [](const char* m) {
+        g_create_err = m;
+        return TP_ERR_INVALID_ARG;
+    };
+    if (n_nodes < 0 || n_out < 0) return bad("n_nodes and n_out must be >= 0");
+    if (n_out > 0 && (!parent || !leaf || !reward || !adv)) return bad("parent, leaf, reward and adv must be non-NULL");
+    if (!workspace || !aligned(workspace, 8) || workspace_bytes < tp::advantage_ws_bytes(n_nodes, n_out))
+        return bad("workspace must be 8-byte aligned and hold tp_advantage_workspace_bytes() bytes");
+    if (stats && !aligned(stats, 8)) return bad("stats must be 8-byte aligned");
+    tp::AdvantageArgs a;
+    a.parent = parent;
+    a.leaf = leaf;
+    a.reward = reward;
+    a.adv = adv;
+    a.stats = stats;
+    a.ws = (uint8_t*)workspace;
+    a.n_nodes = n_nodes;
+    a.n_out = n_out;
+    cudaError_t e = tp::launch_advantage(a, (cudaStream_t)cuda_stream);
+    if (e != cudaSuccess) {
+        g_create_err = std::string("advantage kernel: ") + cudaGetErrorString(e);
+        return TP_ERR_CUDA;
+    }
     return TP_OK;
 }
 
@@ -257,6 +431,7 @@ tp_status tp_fork(tp_tree* t, tp_node node, int32_t k, tp_node* out_children) {
     nd.kids_live += k;
     t->live_nodes += k;
     ++t->version;
+    ++t->struct_version;
     return TP_OK;
 }
 
@@ -277,6 +452,7 @@ tp_status tp_prune(tp_tree* t, tp_node leaf) {
         if (--t->nodes[(size_t)x].kids_live > 0) break;
     }
     ++t->version;
+    ++t->struct_version;
     return TP_OK;
 }
 
@@ -289,12 +465,22 @@ tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void*
     if (!t->cfg.pool) return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree cannot decode");
     if (!Q || !O || !LSE || !aligned(Q, 16) || !aligned(O, 16) || !aligned(LSE, 4))
         return fail(t, TP_ERR_INVALID_ARG, "Q/O must be 16-byte and LSE 4-byte aligned device pointers");
+    // Schedule cache: reuse the last schedule for the same leaf list and
+    // flags; after appends that only filled the leaves' last blocks further
+    // (a decode loop appending one token per leaf), patch its tile words.
     const uint32_t key_flags = flags & ~TP_DECODE_NO_CACHE;
-    const bool hit = !(flags & TP_DECODE_NO_CACHE) && t->sched_valid && t->sched_version == t->version &&
-                     t->sched_flags == key_flags && t->sched_leaves.size() == (size_t)n &&
-                     std::equal(leaves, leaves + n, t->sched_leaves.begin());
+    const bool same_call = !(flags & TP_DECODE_NO_CACHE) && t->sched_valid && t->sched_flags == key_flags &&
+                           t->sched_leaves.size() == (size_t)n &&
+                           std::equal(leaves, leaves + n, t->sched_leaves.begin());
     tp::Schedule& S = t->sched;
-    if (!hit) {
+    if (same_call && t->sched_version != t->version && t->sched_struct == t->struct_version) {
+        tp_status st = patch_cached_schedule(t);
+        if (st != TP_OK) {
+            t->sched_valid = false;
+            return st;
+        }
+        t->sched_version = t->version;
+    } else if (!same_call || t->sched_version != t->version) {
         t->sched_valid = false;
         tp_status st = tp::build_schedule(t, leaves, n, flags, S);
         if (st != TP_OK) return st;
@@ -302,6 +488,7 @@ tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void*
         if (st != TP_OK) return st;
         t->sched_valid = true;
         t->sched_version = t->version;
+        t->sched_struct = t->struct_version;
         t->sched_flags = key_flags;
         t->sched_leaves.assign(leaves, leaves + n);
     }

@@ -78,10 +78,13 @@ static inline int32_t tile_word(int32_t block, int32_t valid) {
 static void node_tiles(const tp_tree* t, const Node& nd, std::vector<int32_t>& tiles) {
     const int32_t bt = t->cfg.block_tokens;
     const int32_t nb = (int32_t)nd.blocks.size();
-    for (int32_t b = 0; b < nb; ++b) {
-        int32_t valid = (b + 1 < nb) ? bt : nd.n_tokens - b * bt;
-        tiles.push_back(tile_word(nd.blocks[(size_t)b], valid));
-    }
+    if (nb == 0) return;
+    const size_t off = tiles.size();
+    tiles.resize(off + (size_t)nb);
+    int32_t* dst = tiles.data() + off;
+    const int32_t* src = nd.blocks.data();
+    for (int32_t b = 0; b < nb; ++b) dst[b] = tile_word(src[b], bt);
+    dst[nb - 1] = tile_word(src[nb - 1], nd.n_tokens - (nb - 1) * bt);
 }
 
 void path_tiles(const tp_tree* t, tp_node leaf, std::vector<int32_t>& tiles) {
@@ -92,15 +95,25 @@ void path_tiles(const tp_tree* t, tp_node leaf, std::vector<int32_t>& tiles) {
 
 // ------------------------------------------------------------ schedule ---
 namespace {
-struct Item {
-    int32_t occ_off;  // into the occ vector
-    int32_t n_occ;
-    int32_t tile_off;  // into the tiles vector
-    int32_t n_tiles;
-};
 constexpr int64_t kTargetUnits = 152 * 2 * 6;  // SMs x resident CTAs x waves
 constexpr int32_t kMinChunkTiles = 4;
 constexpr int32_t kMaxChunkTiles = 64;
+
+// Stable reorder of 8-word unit records by n_tiles, longest first (a
+// counting sort: n_tiles is at most kMaxUnitTiles).
+void sort_units(std::vector<int32_t>& u, std::vector<int32_t>& out, std::vector<int32_t>& bucket) {
+    const size_t cnt = u.size() / kUnitWords;
+    if (cnt < 2) return;
+    bucket.assign(kMaxUnitTiles + 2, 0);
+    for (size_t k = 0; k < cnt; ++k) ++bucket[(size_t)(kMaxUnitTiles - u[k * kUnitWords + U_N_TILES] + 1)];
+    for (int b = 1; b < kMaxUnitTiles + 2; ++b) bucket[(size_t)b] += bucket[(size_t)b - 1];
+    out.resize(u.size());
+    for (size_t k = 0; k < cnt; ++k) {
+        const int32_t pos = bucket[(size_t)(kMaxUnitTiles - u[k * kUnitWords + U_N_TILES])]++;
+        std::memcpy(&out[(size_t)pos * kUnitWords], &u[k * kUnitWords], sizeof(int32_t) * kUnitWords);
+    }
+    u.swap(out);
+}
 }  // namespace
 
 tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t flags, Schedule& S) {
@@ -117,64 +130,99 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
             return fail(t, TP_ERR_EMPTY_PATH, "leaf " + std::to_string(leaves[i]) + " has no token on its path");
     }
 
-    std::vector<Item> items;
-    std::vector<int32_t> occ, tiles;
+    SchedScratch& X = t->scratch;
+    std::vector<Item>& items = X.items;
+    std::vector<int32_t>& occ = X.occ;
+    std::vector<int32_t>& tiles = X.tiles;
+    items.clear();
+    occ.clear();
+    tiles.clear();
+    X.tail_node.clear();
+    X.tail_tile.clear();
+    // a leaf's last tile: recorded when its last block is partly filled,
+    // since only then can an append leave the block list unchanged
+    auto note_tail = [&](const Node& nd, int32_t leaf) {
+        if (!nd.blocks.empty() && nd.n_tokens % t->cfg.block_tokens) {
+            X.tail_node.push_back(leaf);
+            X.tail_tile.push_back((int32_t)tiles.size() - 1);
+        }
+    };
     if (share) {
         // 1. nodes on the union of the paths, with their occurrence counts
         const size_t nn = t->nodes.size();
-        if (t->mark.size() < nn) {
-            t->mark.resize(nn, 0);
-            t->local.resize(nn, 0);
+        if (X.mark.size() < nn) {
+            X.mark.resize(nn, 0);
+            X.local.resize(nn, 0);
         }
-        if (++t->epoch == 0) {
-            std::fill(t->mark.begin(), t->mark.end(), 0u);
-            t->epoch = 1;
+        if (++X.epoch == 0) {
+            std::fill(X.mark.begin(), X.mark.end(), 0u);
+            X.epoch = 1;
         }
-        std::vector<int32_t> touched, cnt;
+        std::vector<int32_t>& touched = X.touched;
+        std::vector<int32_t>& cnt = X.cnt;
+        touched.clear();
+        cnt.clear();
         for (int32_t i = 0; i < n; ++i) {
             for (int32_t x = leaves[i]; x != -1; x = t->nodes[(size_t)x].parent) {
-                if (t->mark[(size_t)x] != t->epoch) {
-                    t->mark[(size_t)x] = t->epoch;
-                    t->local[(size_t)x] = (int32_t)touched.size();
+                if (X.mark[(size_t)x] != X.epoch) {
+                    X.mark[(size_t)x] = X.epoch;
+                    X.local[(size_t)x] = (int32_t)touched.size();
                     touched.push_back(x);
                     cnt.push_back(0);
                 }
-                ++cnt[(size_t)t->local[(size_t)x]];
+                ++cnt[(size_t)X.local[(size_t)x]];
             }
         }
         // 2. occurrence list of every touched node (ascending occurrence)
-        std::vector<int32_t> start(touched.size() + 1, 0), fill(touched.size(), 0), all_occ;
-        for (size_t k = 0; k < touched.size(); ++k) start[k + 1] = start[k] + cnt[k];
-        all_occ.resize((size_t)start.back());
+        const size_t nt = touched.size();
+        X.start.assign(nt + 1, 0);
+        X.fill.assign(nt, 0);
+        for (size_t k = 0; k < nt; ++k) X.start[k + 1] = X.start[k] + cnt[k];
+        X.all_occ.resize((size_t)X.start.back());
         for (int32_t i = 0; i < n; ++i)
             for (int32_t x = leaves[i]; x != -1; x = t->nodes[(size_t)x].parent) {
-                int32_t k = t->local[(size_t)x];
-                all_occ[(size_t)(start[(size_t)k] + fill[(size_t)k]++)] = i;
+                const int32_t k = X.local[(size_t)x];
+                X.all_occ[(size_t)(X.start[(size_t)k] + X.fill[(size_t)k]++)] = i;
             }
         // 3. chains: ids ascend from parent to child, so ascending id order
         //    visits every parent before its children
-        std::vector<int32_t> order(touched);
-        std::sort(order.begin(), order.end());
-        std::vector<int32_t> item_of(touched.size(), -1);
-        std::vector<std::vector<int32_t>> item_nodes;
-        for (int32_t x : order) {
-            const int32_t k = t->local[(size_t)x];
+        X.order.assign(touched.begin(), touched.end());
+        std::sort(X.order.begin(), X.order.end());
+        X.item_of.assign(nt, -1);
+        X.item_cnt.clear();
+        for (int32_t x : X.order) {
+            const int32_t k = X.local[(size_t)x];
             const int32_t p = t->nodes[(size_t)x].parent;
             int32_t it;
-            if (p != -1 && cnt[(size_t)t->local[(size_t)p]] == cnt[(size_t)k]) {
-                it = item_of[(size_t)t->local[(size_t)p]];  // same occurrence set: extend
+            if (p != -1 && cnt[(size_t)X.local[(size_t)p]] == cnt[(size_t)k]) {
+                it = X.item_of[(size_t)X.local[(size_t)p]];  // same occurrence set: extend
             } else {
                 it = (int32_t)items.size();
                 items.push_back({(int32_t)occ.size(), cnt[(size_t)k], 0, 0});
-                occ.insert(occ.end(), all_occ.begin() + start[(size_t)k], all_occ.begin() + start[(size_t)k + 1]);
-                item_nodes.emplace_back();
+                occ.insert(occ.end(), X.all_occ.begin() + X.start[(size_t)k], X.all_occ.begin() + X.start[(size_t)k + 1]);
+                X.item_cnt.push_back(0);
             }
-            item_of[(size_t)k] = it;
-            item_nodes[(size_t)it].push_back(x);
+            X.item_of[(size_t)k] = it;
+            ++X.item_cnt[(size_t)it];
         }
-        for (size_t it = 0; it < items.size(); ++it) {
+        // nodes of each item in ascending id order (CSR)
+        const size_t ni = items.size();
+        X.item_start.assign(ni + 1, 0);
+        for (size_t it = 0; it < ni; ++it) X.item_start[it + 1] = X.item_start[it] + X.item_cnt[it];
+        X.item_nodes.resize(nt);
+        X.fill.assign(ni, 0);
+        for (int32_t x : X.order) {
+            const int32_t it = X.item_of[(size_t)X.local[(size_t)x]];
+            X.item_nodes[(size_t)(X.item_start[(size_t)it] + X.fill[(size_t)it]++)] = x;
+        }
+        for (size_t it = 0; it < ni; ++it) {
             items[it].tile_off = (int32_t)tiles.size();
-            for (int32_t x : item_nodes[it]) node_tiles(t, t->nodes[(size_t)x], tiles);
+            for (int32_t k = X.item_start[it]; k < X.item_start[it + 1]; ++k) {
+                const int32_t x = X.item_nodes[(size_t)k];
+                const Node& nd = t->nodes[(size_t)x];
+                node_tiles(t, nd, tiles);
+                if (nd.state == 0) note_tail(nd, x);
+            }
             items[it].n_tiles = (int32_t)tiles.size() - items[it].tile_off;
         }
     } else {
@@ -183,6 +231,7 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
             Item it{(int32_t)occ.size(), 1, (int32_t)tiles.size(), 0};
             occ.push_back(i);
             path_tiles(t, leaves[i], tiles);
+            note_tail(t->nodes[(size_t)leaves[i]], leaves[i]);
             it.n_tiles = (int32_t)tiles.size() - it.tile_off;
             items.push_back(it);
         }
@@ -199,8 +248,16 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
         kMaxChunkTiles, std::max<int64_t>(kMinChunkTiles, (work + kTargetUnits - 1) / kTargetUnits));
 
     // 5. units, partial slots and merge entries
-    std::vector<int32_t> tc_units, tensor_units, small_units;
-    std::vector<int32_t> pair_occ, pair_slot;  // merge entries before sorting
+    std::vector<int32_t>& tc_units = X.units[0];
+    std::vector<int32_t>& tensor_units = X.units[1];
+    std::vector<int32_t>& small_units = X.units[2];
+    std::vector<int32_t>& pair_occ = X.pair_occ;
+    std::vector<int32_t>& pair_slot = X.pair_slot;
+    tc_units.clear();
+    tensor_units.clear();
+    small_units.clear();
+    pair_occ.clear();
+    pair_slot.clear();
     int32_t n_slots = 0;
     for (const Item& it : items) {
         if (it.n_tiles == 0) continue;
@@ -219,54 +276,52 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
                 pair_occ.push_back(occ[(size_t)(it.occ_off + p)]);
                 pair_slot.push_back(slot_base + p);
             }
-            for (int32_t h = 0; h < hkv; ++h) {
-                if (rows < kTensorMinRows && cuda_core_small) {
-                    const int32_t u[kUnitWords] = {toff, nt, it.occ_off, 0, rows, slot_base, h, KIND_CUDA_CORE};
-                    small_units.insert(small_units.end(), u, u + kUnitWords);
-                } else if (use_tc && (all_tc ? rows >= kTcAnyRows : rows >= kTcMinRows && nt >= kTcMinTiles)) {
-                    for (int32_t r0 = 0; r0 < rows; r0 += kTcRowsPerUnit) {
-                        const int32_t nr = std::min(kTcRowsPerUnit, rows - r0);
-                        const int32_t u[kUnitWords] = {toff, nt, it.occ_off, r0, nr, slot_base, h, KIND_TC};
-                        tc_units.insert(tc_units.end(), u, u + kUnitWords);
-                    }
-                } else {
-                    for (int32_t r0 = 0; r0 < rows; r0 += kTensorRowsPerUnit) {
-                        const int32_t nr = std::min(kTensorRowsPerUnit, rows - r0);
-                        const int32_t u[kUnitWords] = {toff, nt, it.occ_off, r0, nr, slot_base, h, KIND_TENSOR};
-                        tensor_units.insert(tensor_units.end(), u, u + kUnitWords);
-                    }
-                }
+            // one unit per (kv head, block of rows); the kind depends only on
+            // the chunk's rows and length
+            int32_t kind, rpu;
+            if (rows < kTensorMinRows && cuda_core_small) {
+                kind = KIND_CUDA_CORE;
+                rpu = rows;
+            } else if (use_tc && (all_tc ? rows >= kTcAnyRows : rows >= kTcMinRows && nt >= kTcMinTiles)) {
+                kind = KIND_TC;
+                rpu = kTcRowsPerUnit;
+            } else {
+                kind = KIND_TENSOR;
+                rpu = kTensorRowsPerUnit;
             }
+            std::vector<int32_t>& dst = kind == KIND_TC ? tc_units : kind == KIND_TENSOR ? tensor_units : small_units;
+            const int32_t row_blocks = (rows + rpu - 1) / rpu;
+            const size_t at = dst.size();
+            dst.resize(at + (size_t)hkv * row_blocks * kUnitWords);
+            int32_t* u = dst.data() + at;
+            for (int32_t h = 0; h < hkv; ++h)
+                for (int32_t r0 = 0; r0 < rows; r0 += rpu, u += kUnitWords) {
+                    u[U_TILE_OFF] = toff;
+                    u[U_N_TILES] = nt;
+                    u[U_OCC_OFF] = it.occ_off;
+                    u[U_ROW0] = r0;
+                    u[U_N_ROWS] = std::min(rpu, rows - r0);
+                    u[U_SLOT_BASE] = slot_base;
+                    u[U_KVH] = h;
+                    u[U_KIND] = kind;
+                }
             toff += nt;
         }
     }
 
     // 6. unit order: tcgen05, then mma.sync, then CUDA-core units; longer
     //    units first within a kind
-    auto sort_units = [](std::vector<int32_t>& u) {
-        const size_t cnt = u.size() / kUnitWords;
-        std::vector<int32_t> idx(cnt);
-        for (size_t k = 0; k < cnt; ++k) idx[k] = (int32_t)k;
-        std::stable_sort(idx.begin(), idx.end(), [&](int32_t a, int32_t b) {
-            return u[(size_t)a * kUnitWords + U_N_TILES] > u[(size_t)b * kUnitWords + U_N_TILES];
-        });
-        std::vector<int32_t> out(u.size());
-        for (size_t k = 0; k < cnt; ++k)
-            std::memcpy(&out[k * kUnitWords], &u[(size_t)idx[k] * kUnitWords], sizeof(int32_t) * kUnitWords);
-        u.swap(out);
-    };
-    sort_units(tc_units);
-    sort_units(tensor_units);
-    sort_units(small_units);
+    for (auto& u : X.units) sort_units(u, X.sorted, X.bucket);
 
     // 7. merge CSR by occurrence (stable: root-first slot order per leaf)
-    std::vector<int32_t> merge_off((size_t)n + 1, 0), merge_slot(pair_occ.size());
+    std::vector<int32_t>& merge_off = X.merge_off;
+    std::vector<int32_t>& merge_slot = X.merge_slot;
+    merge_off.assign((size_t)n + 1, 0);
+    merge_slot.resize(pair_occ.size());
     for (int32_t i : pair_occ) ++merge_off[(size_t)i + 1];
     for (int32_t i = 0; i < n; ++i) merge_off[(size_t)i + 1] += merge_off[(size_t)i];
-    {
-        std::vector<int32_t> pos(merge_off.begin(), merge_off.end() - 1);
-        for (size_t k = 0; k < pair_occ.size(); ++k) merge_slot[(size_t)pos[(size_t)pair_occ[k]]++] = pair_slot[k];
-    }
+    X.merge_pos.assign(merge_off.begin(), merge_off.end() - 1);
+    for (size_t k = 0; k < pair_occ.size(); ++k) merge_slot[(size_t)X.merge_pos[(size_t)pair_occ[k]]++] = pair_slot[k];
 
     // 8. assemble
     S.n_tc = (int32_t)(tc_units.size() / kUnitWords);
@@ -284,8 +339,9 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     S.off_merge_slot = S.off_merge_off + n + 1;
     const int64_t total = S.off_merge_slot + S.n_merge;
     if (total >= (int64_t)1 << 31) return fail(t, TP_ERR_INVALID_ARG, "schedule too large");
-    S.words.assign((size_t)total, 0);
+    S.words.resize((size_t)total);
     int32_t* w = S.words.data();
+    std::fill(w, w + kSchedHeaderWords, 0);
     w[0] = kSchedMagic;
     w[1] = S.n_units;
     w[2] = S.n_tiles;
@@ -303,7 +359,29 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     std::copy(occ.begin(), occ.end(), w + S.off_occ);
     std::copy(merge_off.begin(), merge_off.end(), w + S.off_merge_off);
     std::copy(merge_slot.begin(), merge_slot.end(), w + S.off_merge_slot);
+    S.leaf_tail.resize(2 * X.tail_node.size());
+    for (size_t k = 0; k < X.tail_node.size(); ++k) {
+        S.leaf_tail[2 * k] = X.tail_node[k];
+        S.leaf_tail[2 * k + 1] = (int32_t)S.off_tiles + X.tail_tile[k];
+    }
     return TP_OK;
+}
+
+int32_t patch_schedule(const tp_tree* t, Schedule& S, std::vector<int32_t>& changed) {
+    changed.clear();
+    const int32_t bt = t->cfg.block_tokens;
+    for (size_t k = 0; k < S.leaf_tail.size(); k += 2) {
+        const Node& nd = t->nodes[(size_t)S.leaf_tail[k]];
+        const int32_t nb = (int32_t)nd.blocks.size();
+        const int32_t word = tile_word(nd.blocks[(size_t)nb - 1], nd.n_tokens - (nb - 1) * bt);
+        int32_t& dst = S.words[(size_t)S.leaf_tail[k + 1]];
+        if (dst != word) {
+            dst = word;
+            changed.push_back(S.leaf_tail[k + 1]);
+            changed.push_back(word);
+        }
+    }
+    return (int32_t)(changed.size() / 2);
 }
 
 }  // namespace tp

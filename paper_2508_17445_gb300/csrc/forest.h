@@ -103,6 +103,48 @@ struct GatherArgs {
     int32_t block_tokens;
 };
 
+// One token per listed node: row i of k / v goes to pool slot slots[i]
+// (block * block_tokens + row).
+struct AppendTokensArgs {
+    const void* k;
+    const void* v;
+    const int32_t* slots;
+    uint8_t* pool;
+    int64_t block_bytes;
+    int32_t head_bytes;
+    int32_t hkv;
+    int32_t n;
+};
+
+// Synthetic activations of the stand-in model (splitmix.h): row i is token
+// (node, pos) with node = row_node ? row_node[i] : node0 and
+// pos = row_node ? pos0 : pos0 + i; each non-null output gets its tag's values.
+struct SynthArgs {
+    uint16_t* k;  // [rows][kv_width]
+    uint16_t* v;  // [rows][kv_width]
+    uint16_t* q;  // [rows][q_width]
+    const int32_t* row_node;
+    uint64_t seed;
+    int64_t rows;
+    int32_t kv_width;
+    int32_t q_width;
+    int32_t node0;
+    int32_t pos0;
+};
+
+// Tree advantage (Eq. tree_ae) over a node table; see tp_tree_advantage.
+struct AdvantageArgs {
+    const int32_t* parent;  // [n_nodes]
+    const int32_t* leaf;    // [n_out]
+    const float* reward;    // [n_out]
+    float* adv;             // [n_out]
+    double* stats;          // [4]: accepted outputs, mean, std, error flag
+    uint8_t* ws;            // workspace, advantage_ws_bytes(n_nodes, n_out)
+    int32_t n_nodes;
+    int32_t n_out;
+};
+int64_t advantage_ws_bytes(int64_t n_nodes, int64_t n_out);
+
 // Launchers (kernels.cu). Return cudaSuccess or the launch error.
 cudaError_t launch_append(int head_dim, const AppendArgs& a, cudaStream_t s);
 // With side != nullptr and both tcgen05 and other units present, the
@@ -112,6 +154,11 @@ cudaError_t launch_decode(int head_dim, const DecodeArgs& a, cudaStream_t s, cud
                           cudaEvent_t fork = nullptr, cudaEvent_t join = nullptr);
 cudaError_t launch_merge(int head_dim, const MergeArgs& a, cudaStream_t s);
 cudaError_t launch_gather(int head_dim, const GatherArgs& a, int64_t n_tokens, cudaStream_t s);
+// sched[pairs[2k]] = pairs[2k + 1] for k < n.
+cudaError_t launch_patch(int32_t* sched, const int32_t* pairs, int32_t n, cudaStream_t s);
+cudaError_t launch_append_tokens(int head_dim, const AppendTokensArgs& a, cudaStream_t s);
+cudaError_t launch_synth(const SynthArgs& a, cudaStream_t s);
+cudaError_t launch_advantage(const AdvantageArgs& a, cudaStream_t s);
 int decode_smem_bytes(int head_dim);
 // Device address of the library's static scratch array (tp_decode_noalloc).
 cudaError_t noalloc_scratch(void** device_ptr);
@@ -145,6 +192,32 @@ struct Schedule {
     std::vector<int32_t> words;  // header | units | tiles | occ | merge_off | merge_slot
     int32_t n_units = 0, n_tiles = 0, n_occ = 0, n = 0, n_slots = 0, n_merge = 0, n_tensor = 0, n_tc = 0;
     int64_t off_units = 0, off_tiles = 0, off_occ = 0, off_merge_off = 0, off_merge_slot = 0;
+    // (leaf node, word index of the last tile of that leaf) for every place a
+    // listed leaf's last block appears: appends that stay inside that block
+    // change only these words (see patch_schedule)
+    std::vector<int32_t> leaf_tail;
+};
+
+// A run of path blocks read with one stacked row set (a node, or a chain of
+// nodes with the same occurrence set).
+struct Item {
+    int32_t occ_off;  // into the occurrence list
+    int32_t n_occ;
+    int32_t tile_off;  // into the tile list
+    int32_t n_tiles;
+};
+
+// Scheduler scratch kept by the tree so repeated schedules reuse their
+// buffers instead of allocating (and page-faulting) fresh ones per call.
+struct SchedScratch {
+    std::vector<uint32_t> mark;   // per node id: epoch of the last visit
+    std::vector<int32_t> local;   // per node id: index among the touched nodes
+    uint32_t epoch = 0;
+    std::vector<int32_t> touched, cnt, start, fill, all_occ, order, item_of, item_cnt, item_start, item_nodes;
+    std::vector<Item> items;
+    std::vector<int32_t> occ, tiles, tail_node, tail_tile;
+    std::vector<int32_t> units[3], sorted, bucket;
+    std::vector<int32_t> pair_occ, pair_slot, merge_off, merge_pos, merge_slot;
 };
 
 }  // namespace tp
@@ -158,10 +231,10 @@ struct tp_tree {
     int64_t live_nodes = 0;
     uint64_t version = 0;  // bumped on every structural change
 
+    uint64_t struct_version = 0;  // bumped on changes other than appends inside a node's last block
+
     // scheduler scratch (reused across calls)
-    std::vector<uint32_t> mark;
-    std::vector<int32_t> local;
-    uint32_t epoch = 0;
+    tp::SchedScratch scratch;
 
     // device scratch owned by the library
     int32_t* d_err = nullptr;  // [0] device error flag, [1..3] decode unit counters
@@ -192,6 +265,15 @@ struct tp_tree {
     tp::Schedule sched;
     bool sched_valid = false;
     uint64_t sched_version = 0;
+    uint64_t sched_struct = 0;  // struct_version the cached schedule was built at
+    std::vector<int32_t> patch_words;
+    int32_t* d_patch = nullptr;
+    int64_t d_patch_cap = 0;
+
+    // tp_append_tokens: pool slot of each appended token
+    std::vector<int32_t> tok_slots;
+    int32_t* d_tok_slots = nullptr;
+    int64_t d_tok_slots_cap = 0;
     uint32_t sched_flags = 0;
     std::vector<int32_t> sched_leaves;
 };
@@ -210,9 +292,23 @@ class LaunchTimer {
     cudaEvent_t b_ = nullptr;
 };
 
+// capi.cpp
+tp_status cuda_fail(tp_tree* t, cudaError_t e, const char* what);
+// Grow a device buffer to at least `need` bytes (contents are not kept);
+// waits for the tree's stream first so no queued kernel still reads it.
+tp_status ensure_device_bytes(tp_tree* t, void** ptr, int64_t* cap, int64_t need, const char* what);
+// Copy `words` int32 words to device `dst` on the tree's stream through a
+// double-buffered pinned staging area; a staging buffer is reused only after
+// its previous copy has completed.
+tp_status stage_upload(tp_tree* t, int32_t* dst, const int32_t* src, int64_t words);
+
 // forest.cpp
 tp_status fail(tp_tree* t, tp_status code, const std::string& msg);
 tp_status check_live(tp_tree* t, tp_node node, bool need_leaf);
 tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t flags, Schedule& out);
+// Refresh the last-tile words of S's leaves from the tree (valid after
+// appends that stayed inside those leaves' last blocks); `changed` receives
+// (word index, new word) pairs. Returns the number of changed words.
+int32_t patch_schedule(const tp_tree* t, Schedule& S, std::vector<int32_t>& changed);
 void path_tiles(const tp_tree* t, tp_node leaf, std::vector<int32_t>& tiles);
 }  // namespace tp

@@ -34,6 +34,7 @@
 #include <mutex>
 
 #include "forest.h"
+#include "splitmix.h"
 
 namespace tp {
 namespace {
@@ -175,6 +176,171 @@ __global__ void append_kernel(const AppendArgs a) {
                        kv_off<kBlockTokens>(row, c);
         *reinterpret_cast<uint4*>(dst) = val;
     }
+}
+
+// ----------------------------------------------------------- token append --
+// Decode-loop append: one token for each of n nodes, each to its own slot.
+template <int HD>
+__global__ void append_tokens_kernel(const AppendTokensArgs a) {
+    constexpr int CH = HD / 8;
+    const int64_t per_kv = (int64_t)a.n * a.hkv * CH;
+    for (int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; idx < 2 * per_kv;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        const int kv = idx >= per_kv;
+        const int64_t r = kv ? idx - per_kv : idx;
+        const int c = (int)(r % CH);
+        const int h = (int)((r / CH) % a.hkv);
+        const int i = (int)(r / ((int64_t)CH * a.hkv));
+        const int32_t slot = a.slots[i];
+        const uint4 val = reinterpret_cast<const uint4*>(kv ? a.v : a.k)[r];
+        uint8_t* dst = a.pool + (int64_t)(slot / kBlockTokens) * a.block_bytes +
+                       (int64_t)(kv * a.hkv + h) * a.head_bytes + kv_off<kBlockTokens>(slot % kBlockTokens, c);
+        *reinterpret_cast<uint4*>(dst) = val;
+    }
+}
+
+// ------------------------------------------------------ stand-in activations --
+// One thread per 64-bit draw = 4 consecutive bf16 values of one row.
+__global__ void synth_kernel(const SynthArgs a) {
+    const int kv_words = a.kv_width / 4, q_words = a.q_width / 4;
+    const int words = (a.k ? kv_words : 0) + (a.v ? kv_words : 0) + (a.q ? q_words : 0);
+    const int64_t total = a.rows * words;
+    for (int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; idx < total;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t i = idx / words;
+        int w = (int)(idx % words);
+        uint16_t* out;
+        uint32_t tag;
+        int width;
+        if (a.k && w < kv_words) {
+            out = a.k, tag = kTagK, width = a.kv_width;
+        } else {
+            if (a.k) w -= kv_words;
+            if (a.v && w < kv_words) {
+                out = a.v, tag = kTagV, width = a.kv_width;
+            } else {
+                if (a.v) w -= kv_words;
+                out = a.q, tag = kTagQ, width = a.q_width;
+            }
+        }
+        const uint32_t node = (uint32_t)(a.row_node ? a.row_node[i] : a.node0);
+        const uint32_t pos = (uint32_t)(a.row_node ? a.pos0 : a.pos0 + i);
+        const uint64_t h = splitmix64(a.seed, draw_counter(tag, node, pos, (uint32_t)w));
+        const uint32_t lo = synth_bf16_bits((uint32_t)h & 0xffffu) | (uint32_t)synth_bf16_bits((uint32_t)(h >> 16) & 0xffffu) << 16;
+        const uint32_t hi = synth_bf16_bits((uint32_t)(h >> 32) & 0xffffu) | (uint32_t)synth_bf16_bits((uint32_t)(h >> 48)) << 16;
+        *reinterpret_cast<uint2*>(out + i * width + 4 * w) = make_uint2(lo, hi);
+    }
+}
+
+// -------------------------------------------------------- tree advantage --
+// Eq. tree_ae over a node table, in one CTA (the tables are small: a few
+// thousand trajectories of a rollout batch). Phases, separated by barriers:
+//   1. every output adds its reward to each strict ancestor's (count, sum)
+//      and folds it into its root's reward range;
+//   2. A_i = mean over those ancestors x of (R_i - sum_x / count_x), for
+//      outputs whose query's rewards are not all equal;
+//   3. mean and (population) std of the A_i over the accepted outputs;
+//   4. adv_i = A_i / std (0 for rejected outputs, or when std is 0).
+constexpr int kAdvThreads = 1024;
+
+__device__ __forceinline__ uint32_t reward_key(float r) {  // order-preserving float -> uint
+    const uint32_t u = __float_as_uint(r);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__device__ double block_sum(double v, double* red) {
+    for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    __syncthreads();
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+    __syncthreads();
+    double s = 0.0;
+    for (int k = 0; k < kAdvThreads / 32; ++k) s += red[k];  // same order in every thread
+    return s;
+}
+
+__global__ void __launch_bounds__(kAdvThreads) advantage_kernel(const AdvantageArgs a) {
+    __shared__ double red[kAdvThreads / 32];
+    __shared__ int bad;
+    const int tid = threadIdx.x;
+    int32_t* cnt = reinterpret_cast<int32_t*>(a.ws);
+    uint32_t* kmin = reinterpret_cast<uint32_t*>(cnt + a.n_nodes);
+    uint32_t* kmax = kmin + a.n_nodes;
+    double* sum = reinterpret_cast<double*>(a.ws + ((12ll * a.n_nodes + 7) / 8) * 8);
+    double* abar = sum + a.n_nodes;
+    int32_t* root_of = reinterpret_cast<int32_t*>(abar + a.n_out);
+    int32_t* depth_of = root_of + a.n_out;
+    if (tid == 0) bad = 0;
+    for (int x = tid; x < a.n_nodes; x += kAdvThreads) {
+        cnt[x] = 0;
+        sum[x] = 0.0;
+        kmin[x] = 0xffffffffu;
+        kmax[x] = 0u;
+    }
+    __syncthreads();
+    for (int i = tid; i < a.n_out; i += kAdvThreads) {
+        const int32_t lf = a.leaf[i];
+        root_of[i] = -1;
+        depth_of[i] = 0;
+        if (lf < 0 || lf >= a.n_nodes) {
+            bad = 1;
+            continue;
+        }
+        const float r = a.reward[i];
+        int32_t root = lf, depth = 0;
+        for (int32_t x = a.parent[lf]; x != -1; x = a.parent[x]) {
+            if (x < -1 || x >= a.n_nodes || depth >= a.n_nodes) {  // malformed table: stop
+                bad = 1;
+                root = -1;
+                break;
+            }
+            atomicAdd(&cnt[x], 1);
+            atomicAdd(&sum[x], (double)r);
+            root = x;
+            ++depth;
+        }
+        if (root < 0) continue;
+        atomicMin(&kmin[root], reward_key(r));
+        atomicMax(&kmax[root], reward_key(r));
+        root_of[i] = root;
+        depth_of[i] = depth;
+    }
+    __syncthreads();
+    double s = 0.0, c = 0.0;
+    for (int i = tid; i < a.n_out; i += kAdvThreads) {
+        const int32_t root = root_of[i], depth = depth_of[i];
+        if (root < 0 || depth == 0 || kmin[root] == kmax[root]) {
+            abar[i] = 0.0;
+            depth_of[i] = 0;  // rejected
+            continue;
+        }
+        const double r = (double)a.reward[i];
+        double acc = 0.0;
+        for (int32_t x = a.parent[a.leaf[i]]; x != -1; x = a.parent[x]) acc += r - sum[x] / (double)cnt[x];
+        abar[i] = acc / (double)depth;
+        s += abar[i];
+        c += 1.0;
+    }
+    const double n_acc = block_sum(c, red);
+    const double mean = n_acc > 0.0 ? block_sum(s, red) / n_acc : 0.0;
+    double v = 0.0;
+    for (int i = tid; i < a.n_out; i += kAdvThreads)
+        if (depth_of[i] > 0) v += (abar[i] - mean) * (abar[i] - mean);
+    const double var = n_acc > 0.0 ? block_sum(v, red) / n_acc : 0.0;
+    const double sd = sqrt(var);
+    for (int i = tid; i < a.n_out; i += kAdvThreads)
+        a.adv[i] = (depth_of[i] > 0 && sd > 0.0) ? (float)(abar[i] / sd) : 0.f;
+    if (tid == 0 && a.stats) {
+        a.stats[0] = n_acc;
+        a.stats[1] = mean;
+        a.stats[2] = sd;
+        a.stats[3] = bad ? 1.0 : 0.0;
+    }
+}
+
+// ------------------------------------------------------- schedule patch --
+__global__ void patch_kernel(int32_t* sched, const int32_t* pairs, int32_t n) {
+    const int k = blockIdx.x * blockDim.x + threadIdx.x;
+    if (k < n) sched[pairs[2 * k]] = pairs[2 * k + 1];
 }
 
 // ------------------------------------------------------------------ gather --
@@ -1682,6 +1848,39 @@ cudaError_t noalloc_scratch(void** device_ptr) {
     }
     *device_ptr = addr[dev];
     return cudaSuccess;
+}
+
+cudaError_t launch_patch(int32_t* sched, const int32_t* pairs, int32_t n, cudaStream_t s) {
+    patch_kernel<<<(n + 255) / 256, 256, 0, s>>>(sched, pairs, n);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append_tokens(int hd, const AppendTokensArgs& a, cudaStream_t s) {
+    const int64_t chunks = 2ll * a.n * a.hkv * (hd / 8);
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((chunks + 255) / 256, 152 * 16));
+    if (hd == 64)
+        append_tokens_kernel<64><<<grid, 256, 0, s>>>(a);
+    else
+        append_tokens_kernel<128><<<grid, 256, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_synth(const SynthArgs& a, cudaStream_t s) {
+    const int64_t words =
+        a.rows * ((a.k ? a.kv_width / 4 : 0) + (a.v ? a.kv_width / 4 : 0) + (a.q ? a.q_width / 4 : 0));
+    if (words == 0) return cudaSuccess;
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((words + 255) / 256, 152 * 16));
+    synth_kernel<<<grid, 256, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+int64_t advantage_ws_bytes(int64_t n_nodes, int64_t n_out) {
+    return ((12 * n_nodes + 7) / 8) * 8 + 8 * n_nodes + 8 * n_out + 8 * n_out;
+}
+
+cudaError_t launch_advantage(const AdvantageArgs& a, cudaStream_t s) {
+    advantage_kernel<<<1, kAdvThreads, 0, s>>>(a);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_append(int hd, const AppendArgs& a, cudaStream_t s) {
