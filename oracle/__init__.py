@@ -18,7 +18,10 @@ Contents
                      append, fork, prune; Sec. 2.2, Algorithm 1), keeps each
                      node's tokens, models the paged pool (fixed-size blocks
                      handed out lowest index first, freed on prune) and
-                     materialises each leaf's root-to-leaf path.
+                     materialises each leaf's root-to-leaf path; ``decode``
+                     and the causal multi-query ``prefill`` (each query sees
+                     its path up to and including itself) run
+                     ``path_attention`` on those paths.
 
 Every function here is pinned by ``tests/test_oracle.py`` against values that
 do not come from this code: a hand-computed two-token example, closed forms,
@@ -233,10 +236,11 @@ class OracleForest:
         return self
 
     # ---- paths --------------------------------------------------------------
-    def path_nodes(self, leaf: int) -> List[int]:
-        """Node ids from the root down to ``leaf``."""
+    def path_nodes(self, leaf: int, any_node: bool = False) -> List[int]:
+        """Node ids from the root down to ``leaf`` (any live node with
+        ``any_node``)."""
         node = self._live(leaf)
-        if node.state != "leaf":
+        if node.state != "leaf" and not any_node:
             raise OracleError("NOT_LEAF", str(leaf))
         out = []
         x = leaf
@@ -254,17 +258,18 @@ class OracleForest:
                 slots.append(node.blocks[t // self.bt] * self.bt + t % self.bt)
         return np.asarray(slots, dtype=np.int64)
 
-    def path_chunks(self, leaf: int) -> List[int]:
+    def path_chunks(self, leaf: int, any_node: bool = False) -> List[int]:
         """kv_ids on the path, root first, in append order."""
         out = []
-        for x in self.path_nodes(leaf):
+        for x in self.path_nodes(leaf, any_node):
             out += self.nodes[x].chunks
         return out
 
-    def path_kv(self, leaf: int, kv_source: Callable[[int], tuple]) -> Tuple[np.ndarray, np.ndarray]:
+    def path_kv(self, leaf: int, kv_source: Callable[[int], tuple],
+                any_node: bool = False) -> Tuple[np.ndarray, np.ndarray]:
         """Materialise the path: K, V as uint16 bf16 bits [N][Hkv][d]."""
         ks, vs = [], []
-        for kv_id in self.path_chunks(leaf):
+        for kv_id in self.path_chunks(leaf, any_node):
             k, v = kv_source(kv_id)
             ks.append(bf16_bits(k))
             vs.append(bf16_bits(v))
@@ -294,6 +299,53 @@ class OracleForest:
         if threads <= 1:
             for i in todo:
                 one(i)
+        else:
+            with ThreadPoolExecutor(max_workers=threads) as ex:
+                list(ex.map(one, todo))
+        return out, lse
+
+    def prefill(self, nodes: Sequence[int], n_queries: Sequence[int], q, kv_source: Callable[[int], tuple],
+                threads: Optional[int] = None, indices: Optional[Sequence[int]] = None):
+        """Causal multi-query attention: fp64 O [sum m][Hq][d], LSE [sum m][Hq].
+
+        The last m_i tokens of nodes[i] are queries (rows of ``q`` packed
+        node by node); query j sits at path position P_i - m_i + j and
+        attends to the path's first P_i - m_i + j + 1 tokens -- the decode
+        definition applied to each prefix of the path.
+        """
+        qb = bf16_bits(q)
+        total = int(sum(n_queries))
+        hq, d = qb.shape[1], qb.shape[2]
+        out = np.full((total, hq, d), np.nan)
+        lse = np.full((total, hq), np.nan)
+        rows = []                                   # (row, node index, visible tokens)
+        r = 0
+        for i, (x, m) in enumerate(zip(nodes, n_queries)):
+            node = self._live(x)
+            path_len = sum(self.nodes[y].n_tokens for y in self.path_nodes(x, True))
+            if m > node.n_tokens:
+                raise OracleError("INVALID_ARG", f"node {x} holds {node.n_tokens} tokens, {m} queries asked")
+            for j in range(m):
+                rows.append((r, i, path_len - m + j + 1))
+                r += 1
+        want = None if indices is None else set(indices)
+        paths: Dict[int, Tuple[np.ndarray, np.ndarray]] = {}
+
+        def one(item):
+            row, i, vis = item
+            if i not in paths:
+                paths[i] = self.path_kv(nodes[i], kv_source, any_node=True)
+            k, v = paths[i]
+            out[row], lse[row] = path_attention(qb[row], k[:vis], v[:vis])
+
+        todo = [it for it in rows if want is None or it[0] in want]
+        for it in todo:                              # materialise paths once, then fan out
+            if it[1] not in paths:
+                paths[it[1]] = self.path_kv(nodes[it[1]], kv_source, any_node=True)
+        threads = threads or min(len(todo), os.cpu_count() or 1) or 1
+        if threads <= 1:
+            for it in todo:
+                one(it)
         else:
             with ThreadPoolExecutor(max_workers=threads) as ex:
                 list(ex.map(one, todo))

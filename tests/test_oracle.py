@@ -323,3 +323,70 @@ def test_empty_path_is_rejected():
     with pytest.raises(oracle.OracleError) as e:
         m.decode([0], torch.zeros(1, 1, 8, dtype=torch.bfloat16), lambda i: None)
     assert e.value.code == "EMPTY_PATH"
+
+
+# --------------------------------------------------------------------------
+# prefill (causal multi-query attention)
+# --------------------------------------------------------------------------
+def _causal_sdpa_rows(k, v, qrows, first_pos, group):
+    """torch fp64 SDPA with an explicit mask: query r (at path position
+    first_pos + r) sees positions <= its own."""
+    n = k.shape[0]
+    m = qrows.shape[0]
+    kk = k.double().permute(1, 0, 2).repeat_interleave(group, dim=0)[None]
+    vv = v.double().permute(1, 0, 2).repeat_interleave(group, dim=0)[None]
+    qq = qrows.double().permute(1, 0, 2)[None]
+    pos = torch.arange(n)[None, :]
+    qpos = (first_pos + torch.arange(m))[:, None]
+    mask = pos <= qpos
+    o = torch.nn.functional.scaled_dot_product_attention(qq, kk, vv, attn_mask=mask)
+    return o[0].permute(1, 0, 2).numpy()
+
+
+def test_prefill_of_single_path_is_causal_sdpa():
+    # one node path of 4 appended chunks; the whole last chunk and then every
+    # token are queries: rows of torch's causal attention
+    s = workloads.single_path(seed=3, lengths=(37, 20, 5, 41), heads=workloads.Heads(6, 2, 64))
+    m = oracle.OracleForest(block_tokens=32).replay(s)
+    leaf = s.leaves[0]
+    k = torch.cat([s.kv(c)[0] for c in range(len(s.kv_len))])
+    v = torch.cat([s.kv(c)[1] for c in range(len(s.kv_len))])
+    n = k.shape[0]
+    node_tokens = m.nodes[leaf].n_tokens
+    gen = torch.Generator().manual_seed(4)
+    for mq in (1, 7, node_tokens):
+        q = torch.randn(mq, 6, 64, generator=gen).to(torch.bfloat16)
+        o, lse = m.prefill([leaf], [mq], q, s.kv)
+        ref = _causal_sdpa_rows(k, v, q, n - mq, 3)
+        np.testing.assert_allclose(o, ref, atol=1e-12)
+
+
+def test_prefill_on_tree_matches_flat_causal_attention_per_node():
+    s = workloads.random_tree(seed=5, n_prompts=2, max_depth=4, heads=workloads.Heads(8, 2, 32))
+    m = oracle.OracleForest(block_tokens=16).replay(s)
+    fwd = _forward_paths(s)
+    live = [x for x, nd in m.nodes.items() if nd.state != "dead" and nd.n_tokens > 0]
+    nodes = live[:6]
+    counts = [min(m.nodes[x].n_tokens, 1 + (3 * i) % 9) for i, x in enumerate(nodes)]
+    gen = torch.Generator().manual_seed(6)
+    q = torch.randn(sum(counts), 8, 32, generator=gen).to(torch.bfloat16)
+    o, lse = m.prefill(nodes, counts, q, s.kv, threads=4)
+    r = 0
+    for x, mq in zip(nodes, counts):
+        chunks = [c for y in m.path_nodes(x, True) for c in m.nodes[y].chunks]
+        k = torch.cat([s.kv(c)[0] for c in chunks])
+        v = torch.cat([s.kv(c)[1] for c in chunks])
+        ref = _causal_sdpa_rows(k, v, q[r:r + mq], k.shape[0] - mq, 4)
+        np.testing.assert_allclose(o[r:r + mq], ref, atol=1e-12)
+        r += mq
+    assert r == len(q) and np.isfinite(lse).all()
+
+
+def test_prefill_of_last_token_equals_decode():
+    s = workloads.tiny(seed=2)
+    m = oracle.OracleForest(block_tokens=32).replay(s)
+    q = s.q()
+    o_d, lse_d = m.decode(s.leaves, q, s.kv)
+    o_p, lse_p = m.prefill(s.leaves, [1] * len(s.leaves), q, s.kv)
+    np.testing.assert_array_equal(o_d, o_p)
+    np.testing.assert_array_equal(lse_d, lse_p)
