@@ -206,6 +206,32 @@ tp_status tp_decode_noalloc(tp_tree* tree, const tp_node* leaves, int32_t n, con
  */
 tp_status tp_append_tokens(tp_tree* tree, const tp_node* nodes, int32_t n, const void* K, const void* V);
 
+/*
+ * Multi-query (prefill) attention over the tree: the last n_queries[i]
+ * tokens of nodes[i] attend causally to that node's root-to-node path --
+ * every ancestor token and the node's own tokens up to and including the
+ * query's position (the segment-level prefill of Sec. 4.3: a segment's
+ * tokens processed together, the shared prefix kept once). Query token j
+ * (0-based) of node i sits at path position P_i - n_queries[i] + j, where P_i
+ * is the node's path length, and sees positions 0 .. that position:
+ *   s_t = q . k_t / sqrt(head_dim) for t <= pos,  LSE = ln sum_t exp(s_t),
+ *   O = sum_t exp(s_t - LSE) v_t.
+ * nodes: host [n] live nodes (leaves or interior, repeats allowed);
+ * n_queries: host [n], 0 <= n_queries[i] <= tokens held by nodes[i]. Q and O:
+ * device bf16 [sum n_queries][num_q_heads][head_dim], rows packed node by
+ * node in token order; LSE: device fp32 [sum n_queries][num_q_heads]. Q, O
+ * 16-byte aligned, LSE 4-byte aligned. Requires num_q_heads / num_kv_heads
+ * <= 64. The work runs as tcgen05 units of up to 128 query rows (whole GQA
+ * groups); flags = TP_PREFILL_MMA_SYNC runs it on the mma.sync path in
+ * 64-row units instead. A row block whose path fits one unit writes O and
+ * LSE directly; longer ones are split and merged by log-sum-exp.
+ * Asynchronous on the tree's stream. Errors: TP_ERR_BAD_NODE,
+ * TP_ERR_INVALID_ARG, TP_ERR_OOM / TP_ERR_CUDA (library scratch).
+ */
+#define TP_PREFILL_MMA_SYNC 32u
+tp_status tp_prefill(tp_tree* tree, const tp_node* nodes, const int32_t* n_queries, int32_t n, const void* Q,
+                     void* O, float* LSE, uint32_t flags);
+
 /* Wait for the tree's stream; TP_ERR_DEVICE if a kernel gave up a bounded
  * wait since the last tp_sync (the flag is then cleared), TP_ERR_CUDA on a
  * CUDA error. */
@@ -453,7 +479,8 @@ tp_status tp_debug_gather(tp_tree* tree, tp_node leaf, void* K_out, void* V_out,
  * small; call with cap 0 to size). Layout:
  *   [0] magic 0x54505344, [1] n_units, [2] n_tiles, [3] n_occ_entries,
  *   [4] n (leaf occurrences), [5] n_slots, [6] n_merge_entries, [7] group g,
- *   [8] n_mma_units, [9] n_tcgen05_units, [10..15] reserved (0),
+ *   [8] n_mma_units, [9] n_tcgen05_units, [10] 0 (1 for prefill schedules),
+ *   [11..15] reserved (0),
  *   then units  [n_units][8]: tile_off, n_tiles, occ_off, row0, n_rows,
  *                             slot_base, kv_head, kind (0 CUDA-core,
  *                             1 mma.sync, 2 tcgen05); tcgen05 units first,
@@ -468,6 +495,15 @@ tp_status tp_debug_gather(tp_tree* tree, tp_node leaf, void* K_out, void* V_out,
  */
 tp_status tp_debug_schedule(tp_tree* tree, const tp_node* leaves, int32_t n, uint32_t flags,
                             int32_t* buf, int64_t cap, int64_t* len);
+
+/* The schedule tp_prefill would run, in the layout above with header word
+ * [10] = 1 and two more sections at the end: unit_pos [n_units] (path
+ * position of each unit's first token) and vis [n] (tokens of its path that
+ * occurrence i -- query token i -- may see). Occurrences are the query
+ * tokens; every unit is an mma.sync unit; a unit row whose occurrence sees
+ * nothing of the unit is computed but has no merge entry. */
+tp_status tp_debug_prefill_schedule(tp_tree* tree, const tp_node* nodes, const int32_t* n_queries, int32_t n,
+                                    uint32_t flags, int32_t* buf, int64_t cap, int64_t* len);
 
 #ifdef __cplusplus
 }

@@ -24,9 +24,9 @@ __all__ = [
     "tp_sync", "tp_last_error", "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop",
     "tp_debug_path", "tp_debug_gather",
     "tp_debug_schedule", "tp_decode_noalloc", "tp_append_tokens", "tp_synth_tokens", "tp_branch_assign",
-    "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "TpRolloutParams", "TpRolloutStats",
+    "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "tp_prefill", "tp_debug_prefill_schedule", "TpRolloutParams", "TpRolloutStats",
     "TpRolloutProbe", "rollout_params", "TP_BRANCH_EVEN", "TP_BRANCH_LOGP_HIGH", "TP_BRANCH_LOGP_LOW",
-    "EVENT_NAMES", "TP_SEG_EOS", "TP_SEG_BOXED", "TP_SEG_FAILED", "TP_SEG_MAX_DEPTH", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE", "TP_DECODE_TCGEN05", "TP_DECODE_ALL_TCGEN05",
+    "EVENT_NAMES", "TP_SEG_EOS", "TP_SEG_BOXED", "TP_SEG_FAILED", "TP_SEG_MAX_DEPTH", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE", "TP_DECODE_TCGEN05", "TP_DECODE_ALL_TCGEN05", "TP_PREFILL_MMA_SYNC",
     "EXPORTED_SYMBOLS",
 ]
 
@@ -39,6 +39,7 @@ TP_DECODE_CUDA_CORE_SMALL = 2
 TP_DECODE_NO_CACHE = 4
 TP_DECODE_TCGEN05 = 8
 TP_DECODE_ALL_TCGEN05 = 16
+TP_PREFILL_MMA_SYNC = 32
 
 TP_BRANCH_EVEN = 0
 TP_BRANCH_LOGP_HIGH = 1
@@ -54,7 +55,8 @@ EXPORTED_SYMBOLS = (
     "tp_append_segment", "tp_fork", "tp_prune", "tp_decode", "tp_decode_ex", "tp_sync", "tp_last_error",
     "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop", "tp_debug_path",
     "tp_debug_gather", "tp_debug_schedule", "tp_decode_noalloc", "tp_append_tokens", "tp_synth_tokens",
-    "tp_branch_assign", "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage",
+    "tp_branch_assign", "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "tp_prefill",
+    "tp_debug_prefill_schedule",
 )
 
 
@@ -150,6 +152,8 @@ def load_library() -> ctypes.CDLL:
         "tp_rollout": (I32, [P, P, P, I64, P, P]),
         "tp_advantage_workspace_bytes": (I64, [I32, I32]),
         "tp_tree_advantage": (I32, [P, I32, P, P, I32, P, P, P, I64, P]),
+        "tp_prefill": (I32, [P, P, P, I32, P, P, P, U32]),
+        "tp_debug_prefill_schedule": (I32, [P, P, P, I32, U32, P, I64, P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -279,17 +283,16 @@ def tp_debug_gather(h, leaf: int, K_out, V_out) -> int:
     return n.value
 
 
-def tp_debug_schedule(h, leaves: Sequence[int], flags: int = 0) -> Dict[str, np.ndarray]:
-    """The schedule tp_decode_ex(flags) would run, decoded into arrays."""
-    arr = _node_array(leaves)
-    lib = load_library()
-    n_words = ctypes.c_int64()
-    _check(h, lib.tp_debug_schedule(h, arr.ctypes.data if len(arr) else None, len(arr), flags, None, 0,
-                                     ctypes.byref(n_words)))
-    buf = np.zeros(max(n_words.value, 1), dtype=np.int32)
-    _check(h, lib.tp_debug_schedule(h, arr.ctypes.data if len(arr) else None, len(arr), flags,
-                                     buf.ctypes.data, len(buf), ctypes.byref(n_words)))
-    w = buf[: n_words.value]
+def tp_prefill(h, nodes: Sequence[int], n_queries: Sequence[int], Q, O, LSE, flags: int = 0) -> None:
+    """Q, O: device bf16 [sum n_queries][Hq][hd]; LSE: device fp32 [sum n_queries][Hq]."""
+    arr = _node_array(nodes)
+    m = np.ascontiguousarray(np.asarray(n_queries, dtype=np.int32).reshape(-1))
+    _check(h, load_library().tp_prefill(h, arr.ctypes.data if len(arr) else None,
+                                        m.ctypes.data if len(m) else None, len(arr), _ptr(Q), _ptr(O), _ptr(LSE),
+                                        flags))
+
+
+def _parse_schedule(w: np.ndarray) -> Dict[str, np.ndarray]:
     assert w[0] == 0x54505344
     n_units, n_tiles, n_occ, n, n_slots, n_merge, g, n_tensor, n_tc = (int(x) for x in w[1:10])
     off = 16
@@ -302,8 +305,39 @@ def tp_debug_schedule(h, leaves: Sequence[int], flags: int = 0) -> Dict[str, np.
     merge_off = w[off: off + n + 1]
     off += n + 1
     merge_slot = w[off: off + n_merge]
-    return {"units": units, "tiles": tiles, "occ": occ, "merge_off": merge_off, "merge_slot": merge_slot,
-            "n_slots": n_slots, "group": g, "n_tensor_units": n_tensor, "n_tc_units": n_tc, "words": w}
+    off += n_merge
+    out = {"units": units, "tiles": tiles, "occ": occ, "merge_off": merge_off, "merge_slot": merge_slot,
+           "n_slots": n_slots, "group": g, "n_tensor_units": n_tensor, "n_tc_units": n_tc, "words": w}
+    if w[10] == 1:
+        out["unit_pos"] = w[off: off + n_units]
+        out["vis"] = w[off + n_units: off + n_units + n]
+    return out
+
+
+def tp_debug_prefill_schedule(h, nodes: Sequence[int], n_queries: Sequence[int], flags: int = 0):
+    """The schedule tp_prefill would run, decoded into arrays."""
+    arr = _node_array(nodes)
+    m = np.ascontiguousarray(np.asarray(n_queries, dtype=np.int32).reshape(-1))
+    lib = load_library()
+    n_words = ctypes.c_int64()
+    args = (arr.ctypes.data if len(arr) else None, m.ctypes.data if len(m) else None, len(arr), flags)
+    _check(h, lib.tp_debug_prefill_schedule(h, *args, None, 0, ctypes.byref(n_words)))
+    buf = np.zeros(max(n_words.value, 1), dtype=np.int32)
+    _check(h, lib.tp_debug_prefill_schedule(h, *args, buf.ctypes.data, len(buf), ctypes.byref(n_words)))
+    return _parse_schedule(buf[: n_words.value])
+
+
+def tp_debug_schedule(h, leaves: Sequence[int], flags: int = 0) -> Dict[str, np.ndarray]:
+    """The schedule tp_decode_ex(flags) would run, decoded into arrays."""
+    arr = _node_array(leaves)
+    lib = load_library()
+    n_words = ctypes.c_int64()
+    _check(h, lib.tp_debug_schedule(h, arr.ctypes.data if len(arr) else None, len(arr), flags, None, 0,
+                                     ctypes.byref(n_words)))
+    buf = np.zeros(max(n_words.value, 1), dtype=np.int32)
+    _check(h, lib.tp_debug_schedule(h, arr.ctypes.data if len(arr) else None, len(arr), flags,
+                                     buf.ctypes.data, len(buf), ctypes.byref(n_words)))
+    return _parse_schedule(buf[: n_words.value])
 
 
 def tp_append_tokens(h, nodes: Sequence[int], K=None, V=None) -> None:

@@ -83,6 +83,8 @@ tp_status ensure_device(tp_tree* t, T*& ptr, int64_t& cap, int64_t need, const c
     return st;
 }
 
+tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O, float* LSE);
+
 tp_status upload_schedule(tp_tree* t, const tp::Schedule& s) {
     const int64_t words = (int64_t)s.words.size();
     tp_status st = ensure_device(t, t->d_sched, t->d_sched_cap, words, "schedule buffer");
@@ -492,12 +494,60 @@ tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void*
         t->sched_flags = key_flags;
         t->sched_leaves.assign(leaves, leaves + n);
     }
+    return run_schedule(t, S, Q, O, LSE);
+}
+
+tp_status tp_prefill(tp_tree* t, const tp_node* nodes, const int32_t* n_queries, int32_t n, const void* Q, void* O,
+                     float* LSE, uint32_t flags) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    if (n < 0) return fail(t, TP_ERR_INVALID_ARG, "n < 0");
+    if (n == 0) return TP_OK;
+    if (!nodes || !n_queries) return fail(t, TP_ERR_INVALID_ARG, "nodes or n_queries is NULL");
+    if (!t->cfg.pool) return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree cannot run attention");
+    if (!Q || !O || !LSE || !aligned(Q, 16) || !aligned(O, 16) || !aligned(LSE, 4))
+        return fail(t, TP_ERR_INVALID_ARG, "Q/O must be 16-byte and LSE 4-byte aligned device pointers");
+    t->sched_valid = false;  // the cached decode schedule's device copy is overwritten
+    tp::Schedule& S = t->sched;
+    tp_status st = tp::build_prefill_schedule(t, nodes, n_queries, n, flags, S);
+    if (st != TP_OK) return st;
+    if (S.n == 0) return TP_OK;
+    st = upload_schedule(t, S);
+    if (st != TP_OK) return st;
+    return run_schedule(t, S, Q, O, LSE);
+}
+
+tp_status tp_debug_prefill_schedule(tp_tree* t, const tp_node* nodes, const int32_t* n_queries, int32_t n,
+                                    uint32_t flags, int32_t* buf, int64_t cap, int64_t* len) {
+    if (!t || !len) return TP_ERR_INVALID_ARG;
+    if (n < 0 || (n > 0 && (!nodes || !n_queries))) return fail(t, TP_ERR_INVALID_ARG, "bad node list");
+    tp::Schedule S;
+    tp_status st = tp::build_prefill_schedule(t, nodes, n_queries, n, flags, S);
+    if (st != TP_OK) return st;
+    *len = (int64_t)S.words.size();
+    if (cap < *len) return cap == 0 ? TP_OK : fail(t, TP_ERR_INVALID_ARG, "buffer too small");
+    if (!buf) return fail(t, TP_ERR_INVALID_ARG, "buf is NULL");
+    std::memcpy(buf, S.words.data(), S.words.size() * 4);
+    return TP_OK;
+}
+
+}  // extern "C"
+
+namespace {
+// Launch the attention and merge kernels of a schedule already on the
+// device (t->d_sched).
+tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O, float* LSE) {
     const int32_t hq = t->cfg.num_q_heads, hd = t->cfg.head_dim;
     const int64_t part_floats = (int64_t)S.n_slots * hq * (hd + 1);
     tp_status st = ensure_device(t, t->d_part, t->d_part_cap, std::max<int64_t>(part_floats, 1), "partial buffer");
     if (st != TP_OK) return st;
 
     tp::DecodeArgs a;
+    if (S.prefill) {
+        a.unit_pos = t->d_sched + S.off_unit_pos;
+        a.vis = t->d_sched + S.off_vis;
+        a.out = (uint16_t*)O;
+        a.out_lse = LSE;
+    }
     a.units = t->d_sched + S.off_units;
     a.tiles = t->d_sched + S.off_tiles;
     a.occ = t->d_sched + S.off_occ;
@@ -539,7 +589,7 @@ tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void*
     m.out = (uint16_t*)O;
     m.lse = LSE;
     m.counters = t->d_err + 1;
-    m.n = n;
+    m.n = S.n_merge > 0 ? S.n : 0;  // 0: every row was written by its only unit; only re-arm the counters
     m.hq = hq;
     {
         tp::LaunchTimer timer(t, tp::KK_MERGE);
@@ -548,6 +598,9 @@ tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void*
     if (e != cudaSuccess) return cuda_fail(t, e, "merge kernel");
     return TP_OK;
 }
+}  // namespace
+
+extern "C" {
 
 tp_status tp_decode_noalloc(tp_tree* t, const tp_node* leaves, int32_t n, const void* Q, void* O, float* LSE,
                             uint32_t flags) {

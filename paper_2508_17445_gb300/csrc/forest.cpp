@@ -99,20 +99,32 @@ constexpr int64_t kTargetUnits = 152 * 2 * 6;  // SMs x resident CTAs x waves
 constexpr int32_t kMinChunkTiles = 4;
 constexpr int32_t kMaxChunkTiles = 64;
 
-// Stable reorder of 8-word unit records by n_tiles, longest first (a
-// counting sort: n_tiles is at most kMaxUnitTiles).
-void sort_units(std::vector<int32_t>& u, std::vector<int32_t>& out, std::vector<int32_t>& bucket) {
-    const size_t cnt = u.size() / kUnitWords;
+// Stable reorder of unit records (`width` words, n_tiles in word
+// U_N_TILES) longest first (a counting sort: n_tiles <= kMaxUnitTiles).
+void sort_units(std::vector<int32_t>& u, std::vector<int32_t>& out, std::vector<int32_t>& bucket,
+                size_t width = kUnitWords) {
+    const size_t cnt = u.size() / width;
     if (cnt < 2) return;
     bucket.assign(kMaxUnitTiles + 2, 0);
-    for (size_t k = 0; k < cnt; ++k) ++bucket[(size_t)(kMaxUnitTiles - u[k * kUnitWords + U_N_TILES] + 1)];
+    for (size_t k = 0; k < cnt; ++k) ++bucket[(size_t)(kMaxUnitTiles - u[k * width + U_N_TILES] + 1)];
     for (int b = 1; b < kMaxUnitTiles + 2; ++b) bucket[(size_t)b] += bucket[(size_t)b - 1];
     out.resize(u.size());
     for (size_t k = 0; k < cnt; ++k) {
-        const int32_t pos = bucket[(size_t)(kMaxUnitTiles - u[k * kUnitWords + U_N_TILES])]++;
-        std::memcpy(&out[(size_t)pos * kUnitWords], &u[k * kUnitWords], sizeof(int32_t) * kUnitWords);
+        const int32_t pos = bucket[(size_t)(kMaxUnitTiles - u[k * width + U_N_TILES])]++;
+        std::memcpy(&out[(size_t)pos * width], &u[k * width], sizeof(int32_t) * width);
     }
     u.swap(out);
+}
+
+// Merge CSR by occurrence from (occurrence, slot) pairs, stable.
+void merge_csr(SchedScratch& X, int32_t n) {
+    X.merge_off.assign((size_t)n + 1, 0);
+    X.merge_slot.resize(X.pair_occ.size());
+    for (int32_t i : X.pair_occ) ++X.merge_off[(size_t)i + 1];
+    for (int32_t i = 0; i < n; ++i) X.merge_off[(size_t)i + 1] += X.merge_off[(size_t)i];
+    X.merge_pos.assign(X.merge_off.begin(), X.merge_off.end() - 1);
+    for (size_t k = 0; k < X.pair_occ.size(); ++k)
+        X.merge_slot[(size_t)X.merge_pos[(size_t)X.pair_occ[k]]++] = X.pair_slot[k];
 }
 }  // namespace
 
@@ -314,14 +326,9 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     for (auto& u : X.units) sort_units(u, X.sorted, X.bucket);
 
     // 7. merge CSR by occurrence (stable: root-first slot order per leaf)
+    merge_csr(X, n);
     std::vector<int32_t>& merge_off = X.merge_off;
     std::vector<int32_t>& merge_slot = X.merge_slot;
-    merge_off.assign((size_t)n + 1, 0);
-    merge_slot.resize(pair_occ.size());
-    for (int32_t i : pair_occ) ++merge_off[(size_t)i + 1];
-    for (int32_t i = 0; i < n; ++i) merge_off[(size_t)i + 1] += merge_off[(size_t)i];
-    X.merge_pos.assign(merge_off.begin(), merge_off.end() - 1);
-    for (size_t k = 0; k < pair_occ.size(); ++k) merge_slot[(size_t)X.merge_pos[(size_t)pair_occ[k]]++] = pair_slot[k];
 
     // 8. assemble
     S.n_tc = (int32_t)(tc_units.size() / kUnitWords);
@@ -364,6 +371,142 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
         S.leaf_tail[2 * k] = X.tail_node[k];
         S.leaf_tail[2 * k + 1] = (int32_t)S.off_tiles + X.tail_tile[k];
     }
+    S.prefill = false;
+    S.off_unit_pos = S.off_vis = 0;
+    return TP_OK;
+}
+
+tp_status build_prefill_schedule(tp_tree* t, const tp_node* nodes, const int32_t* m, int32_t n, uint32_t flags,
+                                 Schedule& S) {
+    const int32_t hq = t->cfg.num_q_heads, hkv = t->cfg.num_kv_heads, g = hq / hkv;
+    if (g > kTensorRowsPerUnit)
+        return fail(t, TP_ERR_INVALID_ARG, "prefill needs num_q_heads / num_kv_heads <= 64");
+    int64_t n_q = 0;
+    for (int32_t i = 0; i < n; ++i) {
+        tp_status st = check_live(t, nodes[i], false);
+        if (st != TP_OK) return st;
+        const Node& nd = t->nodes[(size_t)nodes[i]];
+        if (m[i] < 0 || m[i] > nd.n_tokens)
+            return fail(t, TP_ERR_INVALID_ARG,
+                        "n_queries of node " + std::to_string(nodes[i]) + " must lie in [0, its token count]");
+        n_q += m[i];
+    }
+    if (n_q >= (int64_t)1 << 28) return fail(t, TP_ERR_INVALID_ARG, "too many query tokens in one call");
+    SchedScratch& X = t->scratch;
+    const bool use_tc = !(flags & TP_PREFILL_MMA_SYNC);  // tcgen05 unless asked otherwise (measured faster)
+    const int32_t occ_per_block = (use_tc ? kTcRowsPerUnit : kTensorRowsPerUnit) / g;  // whole GQA groups
+    // path tiles of every listed node, with each tile's path position
+    X.tiles.clear();
+    X.tile_pos.clear();
+    X.node_tile_off.assign((size_t)n + 1, 0);
+    X.vis.resize((size_t)n_q);
+    int64_t work = 0;
+    for (int32_t i = 0, q0 = 0; i < n; q0 += m[i], ++i) {
+        X.node_tile_off[(size_t)i] = (int32_t)X.tiles.size();
+        const size_t first = X.tiles.size();
+        path_tiles(t, nodes[i], X.tiles);
+        int32_t pos = 0;
+        for (size_t k = first; k < X.tiles.size(); ++k) {
+            X.tile_pos.push_back(pos);
+            pos += (X.tiles[k] & ((1 << kTileValidBits) - 1)) + 1;
+        }
+        const Node& nd = t->nodes[(size_t)nodes[i]];
+        const int32_t first_vis = (int32_t)(nd.path_before + nd.n_tokens - m[i]) + 1;
+        for (int32_t o = 0; o < m[i]; ++o) X.vis[(size_t)(q0 + o)] = first_vis + o;
+        for (int32_t o0 = 0; o0 < m[i]; o0 += occ_per_block) {
+            const int32_t o1 = std::min(m[i], o0 + occ_per_block);
+            const int32_t lim = X.vis[(size_t)(q0 + o1 - 1)];
+            const int32_t* tp0 = X.tile_pos.data() + first;
+            work += (int64_t)(std::lower_bound(tp0, tp0 + (X.tiles.size() - first), lim) - tp0) * hkv;
+        }
+    }
+    X.node_tile_off[(size_t)n] = (int32_t)X.tiles.size();
+    const int32_t chunk = (int32_t)std::min<int64_t>(
+        kMaxUnitTiles, std::max<int64_t>(kMinChunkTiles, (work + kTargetUnits - 1) / kTargetUnits));
+
+    // units of 9 words while sorting: the 8 unit words and the path position
+    constexpr int W = kUnitWords + 1;
+    std::vector<int32_t>& recs = X.units[1];
+    recs.clear();
+    X.pair_occ.clear();
+    X.pair_slot.clear();
+    int32_t n_slots = 0;
+    for (int32_t i = 0, q0 = 0; i < n; q0 += m[i], ++i) {
+        const int32_t toff = X.node_tile_off[(size_t)i];
+        const int32_t n_path = X.node_tile_off[(size_t)i + 1] - toff;
+        const int32_t* tpos = X.tile_pos.data() + toff;
+        for (int32_t o0 = 0; o0 < m[i]; o0 += occ_per_block) {
+            const int32_t o1 = std::min(m[i], o0 + occ_per_block);
+            const int32_t lim = X.vis[(size_t)(q0 + o1 - 1)];
+            const int32_t nt = (int32_t)(std::lower_bound(tpos, tpos + n_path, lim) - tpos);  // causal clip
+            const int32_t n_chunks = (nt + chunk - 1) / chunk;
+            const int32_t base = nt / n_chunks, extra = nt % n_chunks;
+            for (int32_t c = 0, t0 = 0; c < n_chunks; ++c) {
+                const int32_t len = base + (c < extra ? 1 : 0);
+                int32_t slot_base = -1;  // one chunk: its units write the final O and LSE
+                if (n_chunks > 1) {
+                    slot_base = n_slots;
+                    n_slots += o1 - o0;
+                    for (int32_t o = o0; o < o1; ++o)
+                        if (X.vis[(size_t)(q0 + o)] > tpos[t0]) {  // the chunk holds tokens this query sees
+                            X.pair_occ.push_back(q0 + o);
+                            X.pair_slot.push_back(slot_base + o - o0);
+                        }
+                }
+                for (int32_t h = 0; h < hkv; ++h) {
+                    const int32_t u[W] = {toff + t0, len, q0 + o0, 0, (o1 - o0) * g, slot_base, h,
+                                          use_tc ? KIND_TC : KIND_TENSOR, tpos[t0]};
+                    recs.insert(recs.end(), u, u + W);
+                }
+                t0 += len;
+            }
+        }
+    }
+    sort_units(recs, X.sorted, X.bucket, W);
+    merge_csr(X, (int32_t)n_q);
+
+    S.prefill = true;
+    S.n_units = (int32_t)(recs.size() / W);
+    S.n_tc = use_tc ? S.n_units : 0;
+    S.n_tensor = use_tc ? 0 : S.n_units;
+    S.n_tiles = (int32_t)X.tiles.size();
+    S.n_occ = (int32_t)n_q;
+    S.n = (int32_t)n_q;
+    S.n_slots = n_slots;
+    S.n_merge = (int32_t)X.merge_slot.size();
+    S.off_units = kSchedHeaderWords;
+    S.off_tiles = S.off_units + (int64_t)S.n_units * kUnitWords;
+    S.off_occ = S.off_tiles + S.n_tiles;
+    S.off_merge_off = S.off_occ + S.n_occ;
+    S.off_merge_slot = S.off_merge_off + S.n + 1;
+    S.off_unit_pos = S.off_merge_slot + S.n_merge;
+    S.off_vis = S.off_unit_pos + S.n_units;
+    const int64_t total = S.off_vis + S.n;
+    if (total >= (int64_t)1 << 31) return fail(t, TP_ERR_INVALID_ARG, "schedule too large");
+    S.words.resize((size_t)total);
+    int32_t* w = S.words.data();
+    std::fill(w, w + kSchedHeaderWords, 0);
+    w[0] = kSchedMagic;
+    w[1] = S.n_units;
+    w[2] = S.n_tiles;
+    w[3] = S.n_occ;
+    w[4] = S.n;
+    w[5] = S.n_slots;
+    w[6] = S.n_merge;
+    w[7] = g;
+    w[8] = S.n_tensor;
+    w[9] = S.n_tc;
+    w[10] = 1;  // prefill schedule
+    for (int32_t k = 0; k < S.n_units; ++k) {
+        std::memcpy(w + S.off_units + (int64_t)k * kUnitWords, &recs[(size_t)k * W], sizeof(int32_t) * kUnitWords);
+        w[S.off_unit_pos + k] = recs[(size_t)k * W + kUnitWords];
+    }
+    std::copy(X.tiles.begin(), X.tiles.end(), w + S.off_tiles);
+    for (int32_t q = 0; q < S.n; ++q) w[S.off_occ + q] = q;
+    std::copy(X.merge_off.begin(), X.merge_off.end(), w + S.off_merge_off);
+    std::copy(X.merge_slot.begin(), X.merge_slot.end(), w + S.off_merge_slot);
+    std::copy(X.vis.begin(), X.vis.end(), w + S.off_vis);
+    S.leaf_tail.clear();
     return TP_OK;
 }
 

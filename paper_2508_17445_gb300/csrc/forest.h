@@ -19,6 +19,9 @@ constexpr int32_t kMaxPoolBlocks = 1 << 24;
 constexpr int kUnitWords = 8;
 enum UnitWord { U_TILE_OFF, U_N_TILES, U_OCC_OFF, U_ROW0, U_N_ROWS, U_SLOT_BASE, U_KVH, U_KIND };
 enum UnitKind { KIND_CUDA_CORE = 0, KIND_TENSOR = 1, KIND_TC = 2 };
+// Launch flavour of tensor units under a causal mask (prefill schedules; the
+// unit words still say KIND_TENSOR).
+constexpr int KIND_PREFILL = 3;
 constexpr int kSchedHeaderWords = 16;
 constexpr int32_t kSchedMagic = 0x54505344;
 // Units with fewer query rows may run on the CUDA-core path
@@ -53,6 +56,10 @@ struct DecodeArgs {
     float* part_o;      // [slot][Hq][hd], normalised partial output
     float* part_lse;    // [slot][Hq], log2-domain partial LSE
     int32_t* err;
+    const int32_t* vis = nullptr;       // prefill: visible path tokens per occurrence (nullptr: decode)
+    const int32_t* unit_pos = nullptr;  // prefill: path position of each unit's first token
+    uint16_t* out = nullptr;            // units with slot_base < 0 write O (bf16 [n][Hq][hd]) and
+    float* out_lse = nullptr;           // LSE (natural log) here directly: their rows have no other part
     int32_t* counters;    // [3] next unit per kind (0 at launch; the merge re-arms them)
     int32_t* counter;     // the counter of the launch in flight (set by the launcher)
     int32_t n_tc_units;      // units [0, n_tc) are tcgen05 units,
@@ -189,9 +196,13 @@ class BlockPool {
 };
 
 struct Schedule {
-    std::vector<int32_t> words;  // header | units | tiles | occ | merge_off | merge_slot
+    // header | units | tiles | occ | merge_off | merge_slot, and for a
+    // prefill schedule also unit_pos [n_units] | vis [n]
+    std::vector<int32_t> words;
     int32_t n_units = 0, n_tiles = 0, n_occ = 0, n = 0, n_slots = 0, n_merge = 0, n_tensor = 0, n_tc = 0;
     int64_t off_units = 0, off_tiles = 0, off_occ = 0, off_merge_off = 0, off_merge_slot = 0;
+    bool prefill = false;
+    int64_t off_unit_pos = 0, off_vis = 0;
     // (leaf node, word index of the last tile of that leaf) for every place a
     // listed leaf's last block appears: appends that stay inside that block
     // change only these words (see patch_schedule)
@@ -218,6 +229,7 @@ struct SchedScratch {
     std::vector<int32_t> occ, tiles, tail_node, tail_tile;
     std::vector<int32_t> units[3], sorted, bucket;
     std::vector<int32_t> pair_occ, pair_slot, merge_off, merge_pos, merge_slot;
+    std::vector<int32_t> tile_pos, node_tile_off, vis;  // prefill
 };
 
 }  // namespace tp
@@ -306,6 +318,13 @@ tp_status stage_upload(tp_tree* t, int32_t* dst, const int32_t* src, int64_t wor
 tp_status fail(tp_tree* t, tp_status code, const std::string& msg);
 tp_status check_live(tp_tree* t, tp_node node, bool need_leaf);
 tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t flags, Schedule& out);
+// Prefill: the last m[i] tokens of nodes[i] attend causally to their root-
+// to-node path. Occurrence q (query token, packed node by node) sees the
+// path's first vis[q] tokens; its rows are kept per node in blocks of whole
+// GQA groups, and each block reads the node's path tiles up to its last
+// visible token, in chunks of at most kMaxUnitTiles tiles.
+tp_status build_prefill_schedule(tp_tree* t, const tp_node* nodes, const int32_t* m, int32_t n, uint32_t flags,
+                                 Schedule& out);
 // Refresh the last-tile words of S's leaves from the tree (valid after
 // appends that stayed inside those leaves' last blocks); `changed` receives
 // (word index, new word) pairs. Returns the number of changed words.

@@ -391,6 +391,7 @@ __global__ void gather_kernel(const GatherArgs a, int64_t n_tokens) {
 // the device error flag and the kernel carries on to a bounded exit.
 struct UnitDesc {
     int tile_off, n_tiles, occ_off, row0, n_rows, slot_base, kvh, kind;
+    int pos0;  // prefill: path position of the unit's first token
 };
 
 template <int HD>
@@ -425,7 +426,7 @@ struct Ctl {
     uint64_t qempty;          // every consumer warp holds its query fragments
     int valid[kStages][2];    // valid tokens of the stage's two tiles (0: no tile)
     int unit[2];              // published unit index (-1: no more units)
-    int desc[2][kUnitWords];  // published unit descriptor
+    int desc[2][kUnitWords + 1];  // published unit descriptor (+ path position)
     int tiles[2][kMaxUnitTiles];  // published unit's tile words
     int abort;
 };
@@ -751,11 +752,14 @@ struct CudaCorePath {
 };
 
 // ---- tensor-core path: 16-row MMA tiles, one per warp -------------------
+// CAUSAL (prefill): row r sees only the first vis[occurrence of r] tokens of
+// its path; the unit's tiles start at path position u.pos0.
 template <int HD>
 struct TensorPath {
     static constexpr int KS = HD / 16;  // k-steps of Q.K^T
     static constexpr int NT = HD / 8;   // n-tiles of the output
 
+    template <bool CAUSAL>
     __device__ static void unit(const DecodeArgs& a, const UnitDesc& u, RingReader& rr, float* park,
                                 const uint8_t* qbuf) {
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -788,11 +792,21 @@ struct TensorPath {
 #pragma unroll
         for (int j = 0; j < NT; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
         float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};  // rows g4, g4 + 8 (lane partial l)
+        int vis[2] = {0, 0}, pos = u.pos0;  // CAUSAL: visible tokens of rows g4, g4 + 8; pair position
+        if constexpr (CAUSAL) {
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int r = mt * 16 + g4 + 8 * h;
+                vis[h] = r < u.n_rows ? a.vis[a.occ[u.occ_off + (u.row0 + r) / a.group]] : 0x7fffffff;
+            }
+        }
 
         const int n_pairs = (u.n_tiles + 1) / 2;
         for (int pr = 0; pr < n_pairs; ++pr) {
             int v0, v1;
             const uint8_t* stage = rr.acquire<HD>(a, v0, v1);
+            const int pos_t0 = pos, pos_t1 = pos + v0;  // path positions of the pair's two tiles
+            pos += v0 + v1;
             if (active) {
                 const uint32_t sk = smem_u32(stage);
                 const uint32_t sv = sk + Smem<HD>::kHalfBytes;
@@ -818,7 +832,10 @@ struct TensorPath {
                         for (int e = 0; e < 4; ++e) {
                             const int tok = tbase + kb + j * 8 + 2 * c4 + (e & 1);
                             const int lim = (tok < kBlockTokens) ? v0 : v1;
-                            const float x = ((tok & 31) < lim) ? s[j][e] * a.qk_scale_log2 : -INFINITY;
+                            bool keep = (tok & 31) < lim;
+                            if constexpr (CAUSAL)
+                                keep = keep && ((tok < kBlockTokens ? pos_t0 : pos_t1) + (tok & 31)) < vis[e >> 1];
+                            const float x = keep ? s[j][e] * a.qk_scale_log2 : -INFINITY;
                             s[j][e] = x;
                             mx[e >> 1] = fmaxf(mx[e >> 1], x);
                         }
@@ -919,10 +936,19 @@ struct TensorPath {
             const int r = mt * 16 + g4 + 8 * h;
             if (r >= u.n_rows) continue;
             const int item_row = u.row0 + r;
-            const int slot = u.slot_base + item_row / a.group;
             const int qh = u.kvh * a.group + item_row % a.group;
-            float* dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
             const float inv = 1.f / l_run[h];
+            if (CAUSAL && u.slot_base < 0) {  // the row's only unit: final O and LSE
+                const int occ = a.occ[u.occ_off + item_row / a.group];
+                uint16_t* dst = a.out + ((int64_t)occ * a.hq + qh) * HD;
+#pragma unroll
+                for (int j = 0; j < NT; ++j)
+                    *reinterpret_cast<uint32_t*>(dst + j * 8 + 2 * c4) = pack_bf16(o[j][2 * h] * inv, o[j][2 * h + 1] * inv);
+                if (c4 == 0) a.out_lse[(int64_t)occ * a.hq + qh] = (m_run[h] + __log2f(l_run[h])) * 0.69314718055994531f;
+                continue;
+            }
+            const int slot = u.slot_base + item_row / a.group;
+            float* dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
 #pragma unroll
             for (int j = 0; j < NT; ++j)
                 *reinterpret_cast<float2*>(dst + j * 8 + 2 * c4) = make_float2(o[j][2 * h] * inv, o[j][2 * h + 1] * inv);
@@ -970,13 +996,14 @@ __device__ void fetch_units(const DecodeArgs& a, Ctl& c, uint8_t* qbuf) {
             dw[U_SLOT_BASE] = d.slot_base;
             dw[U_KVH] = d.kvh;
             dw[U_KIND] = d.kind;
+            dw[kUnitWords] = (u >= 0 && a.unit_pos) ? a.unit_pos[u] : 0;
             *reinterpret_cast<volatile int*>(&c.unit[q]) = u;
         }
         __threadfence_block();  // every lane's tile-word stores, before lane 0 publishes
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&c.ufull[q]));  // release: slot visible to its readers
         if (u < 0) return;
-        if constexpr (KIND == KIND_TENSOR) {
+        if constexpr (KIND == KIND_TENSOR || KIND == KIND_PREFILL) {
             // query rows of the unit: item row row0 + r is q-head
             // kvh * g + (row0 + r) % g of occurrence occ[(row0 + r) / g]
             if (!mbar_wait(smem_u32(&c.qempty), (k & 1) ^ 1)) note_timeout(a, c, 2);
@@ -1047,12 +1074,15 @@ __device__ void consume(const DecodeArgs& a, Ctl& c, uint8_t* ring, float* park,
             d.slot_base = dw[U_SLOT_BASE];
             d.kvh = dw[U_KVH];
             d.kind = dw[U_KIND];
+            d.pos0 = dw[kUnitWords];
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&c.uempty[q]));
         if (u < 0) return;
         if constexpr (KIND == KIND_TENSOR)
-            TensorPath<HD>::unit(a, d, rr, park, qbuf);
+            TensorPath<HD>::template unit<false>(a, d, rr, park, qbuf);
+        else if constexpr (KIND == KIND_PREFILL)
+            TensorPath<HD>::template unit<true>(a, d, rr, park, qbuf);
         else
             CudaCorePath<HD>::unit(a, d, rr, park, scratch);
     }
@@ -1149,7 +1179,7 @@ struct CtlTc {
     uint64_t pv_done;         // a P.V finished (issuer's commit; rescale waits)
     int valid[kStages][2];
     int unit[2];
-    int desc[2][kUnitWords];
+    int desc[2][kUnitWords + 1];  // + path position of the unit's first token (prefill)
     int tiles[2][kMaxUnitTiles];
     int64_t qrow[kTcRows];    // element offset in Q of each row being staged
     uint32_t tmem;
@@ -1201,6 +1231,20 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// the same load without the wait, so two can be in flight
+__device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
+        "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+          "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,"
@@ -1224,6 +1268,7 @@ __device__ __forceinline__ UnitDesc read_desc(const int* slot) {
     d.slot_base = dw[U_SLOT_BASE];
     d.kvh = dw[U_KVH];
     d.kind = dw[U_KIND];
+    d.pos0 = dw[kUnitWords];
     return d;
 }
 
@@ -1250,6 +1295,8 @@ __device__ void tc_fetch(const DecodeArgs& a, CtlTc& c, uint8_t* qbuf) {
         if (u >= 0)
             for (int t = lane; t < n_tiles; t += 32) c.tiles[q][t] = a.tiles[tile_off + t];
         if (lane < kUnitWords) reinterpret_cast<volatile int*>(c.desc[q])[lane] = word;
+        if (lane == kUnitWords)
+            reinterpret_cast<volatile int*>(c.desc[q])[lane] = (u >= 0 && a.unit_pos) ? a.unit_pos[u] : 0;
         if (lane == 0) *reinterpret_cast<volatile int*>(&c.unit[q]) = u;
         __threadfence_block();
         __syncwarp();
@@ -1474,8 +1521,9 @@ __device__ void tc_issue(const DecodeArgs& a, CtlTc& c, const uint8_t* ring, con
     }
 }
 
-// Softmax + epilogue warps: thread = query row (warp * 32 + lane).
-template <int HD>
+// Softmax + epilogue warps: thread = query row (warp * 32 + lane). CAUSAL
+// (prefill): the row sees only the first vis tokens of its path.
+template <int HD, bool CAUSAL>
 __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int row = warp * 32 + lane;
@@ -1493,10 +1541,19 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
         const volatile int* tw = c.tiles[q];
         const int n_pairs = (d.n_tiles + 1) / 2;
         float m_used = -INFINITY, l = 0.f;
+        int vis = 0x7fffffff, pos = d.pos0;
+        if (CAUSAL && row < d.n_rows) vis = a.vis[a.occ[d.occ_off + (d.row0 + row) / a.group]];
         for (int j = 0; j < n_pairs; ++j) {
             const uint32_t g_stage = gs + j, sb = g_stage & 1;
             const int v0 = (tw[2 * j] & ((1 << kTileValidBits) - 1)) + 1;
             const int v1 = 2 * j + 1 < d.n_tiles ? (tw[2 * j + 1] & ((1 << kTileValidBits) - 1)) + 1 : 0;
+            // CAUSAL: tokens of tile h visible to this row: lim_h = min(valid, vis - position)
+            int lim0 = v0, lim1 = v1;
+            if (CAUSAL) {
+                lim0 = max(0, min(v0, vis - pos));
+                lim1 = max(0, min(v1, vis - (pos + v0)));
+                pos += v0 + v1;
+            }
             if (!mbar_wait(smem_u32(&c.s_full[sb]), (g_stage >> 1) & 1)) note_timeout(a, c, 1);
             tc_fence_after();
             if (warp * 32 >= d.n_rows) {  // padding rows only: their P is never read back
@@ -1505,16 +1562,19 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
                 continue;
             }
             const uint32_t s_addr = lane_addr + sb * kStageTokens;
-            uint32_t r[32];
-            // pass 1: row max over the stage's valid tokens
+            // the stage's 64 scores of this row, read once (two loads in flight)
+            uint32_t r[2][32];
+            tmem_ld32_nowait(s_addr, r[0]);
+            tmem_ld32_nowait(s_addr + 32, r[1]);
+            tmem_wait_ld();
+            // row max over the tokens the row may see
             float mx = -INFINITY;
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
-                tmem_ld32(s_addr + h * 32, r);
-                const int lim = h ? v1 : v0;
+                const int lim = h ? lim1 : lim0;
 #pragma unroll
                 for (int t = 0; t < 32; ++t)
-                    if (t < lim) mx = fmaxf(mx, __uint_as_float(r[t]) * a.qk_scale_log2);
+                    if (t < lim) mx = fmaxf(mx, __uint_as_float(r[h][t]) * a.qk_scale_log2);
             }
             const float m_new = fmaxf(m_used, mx);
             const bool need = m_new > m_used + kRescaleLog2;
@@ -1537,17 +1597,17 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
                     m_used = m_new;
                 }
             }
-            // pass 2: P = exp2(s - m_used) as bf16 pairs over the S columns
+            // P = exp2(s - m_used) as bf16 pairs over the S columns
             uint32_t pw[32];
             float sum = 0.f;
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
-                tmem_ld32(s_addr + h * 32, r);
-                const int lim = h ? v1 : v0;
+                const int lim = h ? lim1 : lim0;
 #pragma unroll
                 for (int t = 0; t < 32; t += 2) {
-                    const float p0 = t < lim ? fast_exp2(__uint_as_float(r[t]) * a.qk_scale_log2 - m_used) : 0.f;
-                    const float p1 = t + 1 < lim ? fast_exp2(__uint_as_float(r[t + 1]) * a.qk_scale_log2 - m_used) : 0.f;
+                    const float p0 = t < lim ? fast_exp2(__uint_as_float(r[h][t]) * a.qk_scale_log2 - m_used) : 0.f;
+                    const float p1 =
+                        t + 1 < lim ? fast_exp2(__uint_as_float(r[h][t + 1]) * a.qk_scale_log2 - m_used) : 0.f;
                     sum += p0 + p1;
                     pw[h * 16 + t / 2] = pack_bf16(p0, p1);
                 }
@@ -1571,25 +1631,42 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
             continue;
         }
         const bool live = row < d.n_rows;
+        const bool final_out = CAUSAL && d.slot_base < 0;  // the row's only unit: final O and LSE
         float* dst = nullptr;
+        uint16_t* dst16 = nullptr;
         if (live) {
             const int item_row = d.row0 + row;
-            const int slot = d.slot_base + item_row / a.group;
             const int qh = d.kvh * a.group + item_row % a.group;
-            dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
-            a.part_lse[(int64_t)slot * a.hq + qh] = m_used + __log2f(l);
+            if (final_out) {
+                const int occ = a.occ[d.occ_off + item_row / a.group];
+                dst16 = a.out + ((int64_t)occ * a.hq + qh) * HD;
+                a.out_lse[(int64_t)occ * a.hq + qh] = (m_used + __log2f(l)) * 0.69314718055994531f;
+            } else {
+                const int slot = d.slot_base + item_row / a.group;
+                dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
+                a.part_lse[(int64_t)slot * a.hq + qh] = m_used + __log2f(l);
+            }
         }
         const float inv = 1.f / l;
 #pragma unroll 1
         for (int cc = 0; cc < HD / 32; ++cc) {
             uint32_t ov[32];
             tmem_ld32(o_addr + cc * 32, ov);
-            if (live)
+            if (live && final_out) {
+#pragma unroll
+                for (int t = 0; t < 32; t += 8)
+                    *reinterpret_cast<uint4*>(dst16 + cc * 32 + t) =
+                        make_uint4(pack_bf16(__uint_as_float(ov[t]) * inv, __uint_as_float(ov[t + 1]) * inv),
+                                   pack_bf16(__uint_as_float(ov[t + 2]) * inv, __uint_as_float(ov[t + 3]) * inv),
+                                   pack_bf16(__uint_as_float(ov[t + 4]) * inv, __uint_as_float(ov[t + 5]) * inv),
+                                   pack_bf16(__uint_as_float(ov[t + 6]) * inv, __uint_as_float(ov[t + 7]) * inv));
+            } else if (live) {
 #pragma unroll
                 for (int t = 0; t < 32; t += 4)
                     *reinterpret_cast<float4*>(dst + cc * 32 + t) =
                         make_float4(__uint_as_float(ov[t]) * inv, __uint_as_float(ov[t + 1]) * inv,
                                     __uint_as_float(ov[t + 2]) * inv, __uint_as_float(ov[t + 3]) * inv);
+            }
         }
         tc_fence_before();
         __syncwarp();
@@ -1600,7 +1677,7 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
     }
 }
 
-template <int HD>
+template <int HD, bool CAUSAL>
 __global__ void __launch_bounds__(kTcThreads, 2) decode_tc_kernel(const DecodeArgs a) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     __shared__ __align__(16) CtlTc ctl;
@@ -1644,7 +1721,7 @@ __global__ void __launch_bounds__(kTcThreads, 2) decode_tc_kernel(const DecodeAr
     __syncthreads();
     tc_fence_after();
     if (warp < kTcConsumerWarps)
-        tc_consume<HD>(a, ctl);
+        tc_consume<HD, CAUSAL>(a, ctl);
     else if (warp == kTcStreamerWarp) {
         if ((tid & 31) == 0) tc_stream<HD>(a, ctl, ring);
     } else if (warp == kTcFetcherWarp)
@@ -1667,6 +1744,7 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
     if (warp_global >= a.n * a.hq) return;
     const int i = warp_global / a.hq, qh = warp_global % a.hq;
     const int beg = a.merge_off[i], ns = a.merge_off[i + 1] - beg;
+    if (ns == 0) return;  // written directly by its only unit
     float acc[DPL];
 #pragma unroll
     for (int d = 0; d < DPL; ++d) acc[d] = 0.f;
@@ -1767,16 +1845,16 @@ cudaError_t launch_range(DecodeArgs a, int begin, int end, int32_t* counter, cud
     return cudaGetLastError();
 }
 
-template <int HD>
+template <int HD, bool CAUSAL>
 int decode_tc_grid() {
     static int grid = [] {
         int dev = 0, sms = 0, per_sm = 0;
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        if (cudaFuncSetAttribute(decode_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        if (cudaFuncSetAttribute(decode_tc_kernel<HD, CAUSAL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  TcSmem<HD>::kBytes) != cudaSuccess)
             return 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_tc_kernel<HD>, kTcThreads,
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_tc_kernel<HD, CAUSAL>, kTcThreads,
                                                           TcSmem<HD>::kBytes) != cudaSuccess)
             return 0;
         // each resident CTA holds kTmemCols of the SM's 512 tensor-memory columns
@@ -1788,12 +1866,16 @@ int decode_tc_grid() {
 template <int HD>
 cudaError_t launch_tc_range(DecodeArgs a, int begin, int end, int32_t* counter, cudaStream_t s) {
     if (end <= begin) return cudaSuccess;
-    const int slots = decode_tc_grid<HD>();
+    const bool causal = a.vis != nullptr;
+    const int slots = causal ? decode_tc_grid<HD, true>() : decode_tc_grid<HD, false>();
     if (slots == 0) return cudaErrorInvalidConfiguration;
     a.unit_begin = begin;
     a.unit_end = end;
     a.counter = counter;
-    decode_tc_kernel<HD><<<std::min(end - begin, slots), kTcThreads, TcSmem<HD>::kBytes, s>>>(a);
+    if (causal)
+        decode_tc_kernel<HD, true><<<std::min(end - begin, slots), kTcThreads, TcSmem<HD>::kBytes, s>>>(a);
+    else
+        decode_tc_kernel<HD, false><<<std::min(end - begin, slots), kTcThreads, TcSmem<HD>::kBytes, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -1812,7 +1894,8 @@ cudaError_t launch_decode_hd(const DecodeArgs& a, cudaStream_t s, cudaStream_t s
         e = launch_tc_range<HD>(a, 0, tc_end, a.counters, s);
     }
     if (e != cudaSuccess) return e;
-    e = launch_range<HD, KIND_TENSOR>(a, tc_end, mma_end, a.counters + 1, s);
+    e = a.vis ? launch_range<HD, KIND_PREFILL>(a, tc_end, mma_end, a.counters + 1, s)
+              : launch_range<HD, KIND_TENSOR>(a, tc_end, mma_end, a.counters + 1, s);
     if (e != cudaSuccess) return e;
     e = launch_range<HD, KIND_CUDA_CORE>(a, mma_end, a.n_units, a.counters + 2, s);
     if (e != cudaSuccess) return e;
@@ -1911,8 +1994,7 @@ cudaError_t launch_decode(int hd, const DecodeArgs& a, cudaStream_t s, cudaStrea
 
 cudaError_t launch_merge(int hd, const MergeArgs& a, cudaStream_t s) {
     const int64_t warps = (int64_t)a.n * a.hq;
-    if (warps == 0) return cudaSuccess;
-    const int grid = (int)((warps + 3) / 4);
+    const int grid = (int)std::max<int64_t>(1, (warps + 3) / 4);  // one block at least: it re-arms the counters
     if (hd == 64)
         merge_kernel<64><<<grid, 128, 0, s>>>(a);
     else

@@ -369,6 +369,23 @@ def shared_prompt(seed: int = 0, prompt: int = 2000, n_leaves: int = 3, leaf_tok
                   f"prompt {prompt} shared by {n_leaves} leaves")
 
 
+def segment_prefill(seed: int = 0, n_prompts: int = 4, prompt_len: int = 1024, fanout: int = 4,
+                    seg_len: int = 512, heads: Heads = Heads(28, 4, 128)) -> Script:
+    """Prefill shape: each prompt forked into `fanout` leaves that each hold
+    a freshly appended segment of `seg_len` tokens (the tokens a prefill
+    call processes as queries, Sec. 4.3)."""
+    b = _Builder()
+    leaves = []
+    for _ in range(n_prompts):
+        r = b.root()
+        b.append(r, prompt_len)
+        for c in b.fork(r, fanout):
+            b.append(c, seg_len)
+            leaves.append(c)
+    return Script("segment_prefill", heads, seed, b.ops, leaves, b.kv_len,
+                  f"{n_prompts} prompts of {prompt_len} tokens x {fanout} leaves of {seg_len}-token segments")
+
+
 CONFIG_NAMES = ("tiny", "qwen7b", "random_divergence", "wide_prefix", "no_sharing")
 
 
