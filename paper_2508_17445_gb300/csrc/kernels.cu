@@ -1857,6 +1857,19 @@ int decode_tc_grid() {
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_tc_kernel<HD, CAUSAL>, kTcThreads,
                                                           TcSmem<HD>::kBytes) != cudaSuccess)
             return 0;
+        // The occupancy query answers 1 for this kernel on GB300 although its
+        // registers (128 x 224 threads) and shared memory fit twice per SM, so
+        // count from those resources too. Launching more CTAs than fit is
+        // harmless for a persistent kernel: a CTA that starts late finds the
+        // unit counter exhausted and exits.
+        cudaFuncAttributes fa{};
+        int smem_sm = 0, reserved = 0;
+        if (cudaFuncGetAttributes(&fa, decode_tc_kernel<HD, CAUSAL>) != cudaSuccess) return 0;
+        cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
+        cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev);
+        const int by_smem = smem_sm / (int)(TcSmem<HD>::kBytes + fa.sharedSizeBytes + reserved);
+        const int by_regs = 65536 / (fa.numRegs * kTcThreads);
+        per_sm = std::max(per_sm, std::min(by_smem, by_regs));
         // each resident CTA holds kTmemCols of the SM's 512 tensor-memory columns
         return sms * std::min(std::max(per_sm, 1), 512 / (int)kTmemCols);
     }();
