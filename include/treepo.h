@@ -155,12 +155,15 @@ tp_status tp_decode(tp_tree* tree, const tp_node* leaves, int32_t n, const void*
                                       /* path (default: tensor cores, rows padded to */
                                       /* one 16-row MMA tile)                        */
 #define TP_DECODE_NO_CACHE 4u         /* rebuild the schedule even if cached         */
-#define TP_DECODE_TCGEN05 8u          /* chunks of >= 64 stacked rows and >= 32      */
-                                      /* blocks on tcgen05 (128-row units, running   */
-                                      /* concurrently with the rest)                 */
-#define TP_DECODE_ALL_TCGEN05 16u     /* every unit of > 16 stacked rows on tcgen05  */
-                                      /* Default: all stacked rows on mma.sync in    */
-                                      /* 64-row blocks (measured faster on GB300).   */
+#define TP_DECODE_TCGEN05 8u          /* tcgen05 only for chunks of >= 64 stacked    */
+                                      /* rows and >= 32 blocks; the other stacked    */
+                                      /* rows on mma.sync in 64-row units            */
+#define TP_DECODE_ALL_TCGEN05 16u     /* the default: every unit of > 16 stacked     */
+                                      /* rows on tcgen05 (128-row units, running     */
+                                      /* concurrently with the mma.sync units of one */
+                                      /* 16-row tile; measured fastest on GB300)     */
+#define TP_MMA_SYNC 32u               /* no tcgen05: stacked rows on mma.sync in     */
+                                      /* 64-row units (decode and tp_prefill)        */
 tp_status tp_decode_ex(tp_tree* tree, const tp_node* leaves, int32_t n, const void* Q, void* O,
                        float* LSE, uint32_t flags);
 
@@ -222,13 +225,12 @@ tp_status tp_append_tokens(tp_tree* tree, const tp_node* nodes, int32_t n, const
  * node in token order; LSE: device fp32 [sum n_queries][num_q_heads]. Q, O
  * 16-byte aligned, LSE 4-byte aligned. Requires num_q_heads / num_kv_heads
  * <= 64. The work runs as tcgen05 units of up to 128 query rows (whole GQA
- * groups); flags = TP_PREFILL_MMA_SYNC runs it on the mma.sync path in
- * 64-row units instead. A row block whose path fits one unit writes O and
+ * groups); flags = TP_MMA_SYNC runs it on the mma.sync path in 64-row
+ * units instead. A row block whose path fits one unit writes O and
  * LSE directly; longer ones are split and merged by log-sum-exp.
  * Asynchronous on the tree's stream. Errors: TP_ERR_BAD_NODE,
  * TP_ERR_INVALID_ARG, TP_ERR_OOM / TP_ERR_CUDA (library scratch).
  */
-#define TP_PREFILL_MMA_SYNC 32u
 tp_status tp_prefill(tp_tree* tree, const tp_node* nodes, const int32_t* n_queries, int32_t n, const void* Q,
                      void* O, float* LSE, uint32_t flags);
 
@@ -303,8 +305,8 @@ tp_status tp_branch_assign(const double* logp, int32_t n, int32_t budget, int32_
  *   mix(seed + (ctr + 1) * 0x9E3779B97F4A7C15),
  *   ctr = tag << 60 | a << 32 | b << 12 | c   (a < 2^28, b < 2^20, c < 2^12),
  * read as u = (x >> 11) * 2^-53 in [0, 1) for decisions, or as four bf16
- * values (16 bits each, low bits first: sign bit 15, exponent 125 + bits
- * 7..8, mantissa bits 0..6; values in +-[0.25, 4)) for activations:
+ * values (16 bits each, low bits first: sign bit 15, exponent 124 + bits
+ * 7..8, mantissa bits 0..6; values in +-[0.125, 2)) for activations:
  *   K, V, Q of token b of node a: tags 1, 2, 3, c = word of the row
  *       ([heads][head_dim] row-major, 4 values per word);
  *   token b of segment node a is EOS if u(4, a, b, 0) < p_eos (the segment

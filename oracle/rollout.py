@@ -80,8 +80,9 @@ def synth_rows(seed: int, tag: int, nodes: Sequence[int], positions: Sequence[in
                head_dim: int) -> np.ndarray:
     """Stand-in activations: bf16 bit patterns [rows][heads][head_dim] of
     token (nodes[i], positions[i]). Each 64-bit draw gives four values, low
-    16 bits first; 16 bits r give sign r[15], exponent 125 + r[7:9] and
-    mantissa r[0:7], i.e. values in +-[0.25, 4)."""
+    16 bits first; 16 bits r give sign r[15], exponent 124 + r[7:9] and
+    mantissa r[0:7], i.e. values in +-[0.125, 2) -- root mean square about
+    0.9, the scale of the unit-normal inputs of the decode workloads."""
     width = heads * head_dim
     words = width // 4
     node = np.asarray(nodes, dtype=np.uint64)[:, None]
@@ -92,7 +93,7 @@ def synth_rows(seed: int, tag: int, nodes: Sequence[int], positions: Sequence[in
     h = _splitmix64_np(seed, ctr)                                          # [rows][words]
     lanes = np.stack([(h >> np.uint64(16 * k)) & np.uint64(0xFFFF) for k in range(4)], axis=-1)
     r = lanes.astype(np.uint32)
-    bits = (r & 0x8000) | ((125 + ((r >> 7) & 3)) << 7) | (r & 0x7F)
+    bits = (r & 0x8000) | ((124 + ((r >> 7) & 3)) << 7) | (r & 0x7F)
     return bits.astype(np.uint16).reshape(len(nodes), heads, head_dim)
 
 

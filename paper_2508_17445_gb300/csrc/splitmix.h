@@ -49,9 +49,10 @@ TP_HD double draw_uniform(uint64_t seed, uint32_t tag, uint32_t a, uint32_t b, u
 }
 
 // bf16 bit pattern from 16 random bits: random sign and 7-bit mantissa,
-// exponent 2^-2 .. 2^1, so values lie in +-[0.25, 4).
+// exponent 2^-3 .. 2^0, so values lie in +-[0.125, 2) (root mean square
+// about 0.9, the scale of unit-normal activations).
 TP_HD uint16_t synth_bf16_bits(uint32_t r16) {
-    return (uint16_t)((r16 & 0x8000u) | ((125u + ((r16 >> 7) & 3u)) << 7) | (r16 & 0x7fu));
+    return (uint16_t)((r16 & 0x8000u) | ((124u + ((r16 >> 7) & 3u)) << 7) | (r16 & 0x7fu));
 }
 
 }  // namespace tp

@@ -42,15 +42,18 @@ def test_synth_rows_bit_layout():
     bits = R.synth_rows(5, R.TAG_K, [3, 3, 9], [0, 1, 0], 2, 8)
     assert bits.shape == (3, 2, 8) and bits.dtype == np.uint16
     vals = np.abs(R.bf16_to_f64(bits))
-    assert vals.min() >= 0.25 and vals.max() < 4.0
+    assert vals.min() >= 0.125 and vals.max() < 2.0
     # word 1 of row (node 3, token 1) holds elements 4..7, low 16 bits first
     h = R.splitmix64(5, R.counter(R.TAG_K, 3, 1, 1))
     for lane in range(4):
         r = (h >> (16 * lane)) & 0xFFFF
-        sign, expo, mant = r >> 15, 125 + ((r >> 7) & 3), r & 0x7F
+        sign, expo, mant = r >> 15, 124 + ((r >> 7) & 3), r & 0x7F
         assert R.bf16_to_f64(bits[1:2, 0, 4 + lane])[0] == (-1) ** sign * 2.0 ** (expo - 127) * (1 + mant / 128)
     big = R.bf16_to_f64(R.synth_rows(1, R.TAG_V, list(range(64)), [7] * 64, 4, 64))
     assert abs((big > 0).mean() - 0.5) < 0.03
+    # unit-normal scale: E[x^2] = E[(1 + m)^2] * mean(4^e), e in -3..0, m uniform on [0, 1)
+    want_ms = (7 / 3) * (4.0 ** -3 + 4.0 ** -2 + 4.0 ** -1 + 1) / 4
+    assert abs((big ** 2).mean() - want_ms) < 0.05 * want_ms
 
 
 # ---------------------------------------------------------- branch split --
