@@ -34,6 +34,7 @@ METRIC = "tree-decode leaf-queries/s; HBM GB/s on unique KV bytes vs GB300 peak"
 UNIT = "leaf-queries/s"
 DEFAULT_WORKLOAD = "qwen7b"
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
 
 
 def parse():
@@ -42,7 +43,11 @@ def parse():
     p.add_argument("--steps", type=int, default=20)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--workload", default=DEFAULT_WORKLOAD,
-                   choices=["tiny", "qwen7b", "random_divergence", "wide_prefix", "no_sharing"])
+                   choices=["tiny", "qwen7b", "random_divergence", "wide_prefix", "no_sharing", "rollout", "prefill",
+                            "advantage"],
+                   help="a decode forest (the default line), or one of the other measured paths: rollout "
+                        "(Algorithm 1 with decode after every token), prefill (causal multi-query attention), "
+                        "advantage (Eq. tree_ae)")
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--prompts", type=int, default=None,
                    help="scale the workload down to this many prompts (small cases for ncu captures)")
@@ -117,14 +122,14 @@ def workload_label(script):
     return f"{script.name}: {script.description}; {h.num_q_heads} q / {h.num_kv_heads} kv heads, head_dim {h.head_dim}, bf16"
 
 
-def peaks():
+def peaks(key="hbm_gbs"):
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
         with open(path) as f:
             d = json.load(f)
-        return float(d["hbm_gbs"]), "measured"
+        return float(d[key]), "measured"
     except Exception:
-        return FALLBACK_HBM_GBS, "fallback"
+        return (FALLBACK_HBM_GBS if key == "hbm_gbs" else FALLBACK_BF16_TFLOPS), "fallback"
 
 
 def kernel_source_hash():
@@ -293,6 +298,396 @@ def run_reference(args, rank, world):
 
 
 # --------------------------------------------------------------------------
+# the other paths: rollout driver, prefill attention, tree advantage
+# --------------------------------------------------------------------------
+ROLLOUT_SHAPE = dict(n_prompts=64, width=16, max_depth=14, seg_tokens=512, init_branches=2, p_eos=1 / 2048,
+                     p_boxed=0.03, p_fail=0.03, p_correct=0.5)
+
+
+def rollout_prompts(n, seed):
+    import numpy as np
+    return [int(x) for x in np.random.default_rng(seed).integers(256, 1025, n)]
+
+
+def rollout_decode_bytes(events, heads):
+    """Algorithmic bytes of every decode call of a rollout run with decode on,
+    from its events: per call, the unique K/V tokens of the paths still
+    generating (their leaf holding t + 1 tokens at token step t) plus their
+    query rows."""
+    EV_ROOT, EV_FORK, EV_SEGMENT = 1, 2, 3
+    parent, tok = {}, {}
+    kv_tok = 2 * heads.num_kv_heads * heads.head_dim * 2
+    q_row = heads.num_q_heads * heads.head_dim * 2
+    total = rows = 0
+    i, n = 0, len(events)
+    while i < n:
+        kind = int(events[i][0])
+        if kind == EV_ROOT:
+            parent[int(events[i][2])] = -1
+            tok[int(events[i][2])] = int(events[i][3])
+            i += 1
+        elif kind == EV_FORK:
+            for c in range(int(events[i][3]), int(events[i][3]) + int(events[i][4])):
+                parent[c] = int(events[i][2])
+            i += 1
+        elif kind == EV_SEGMENT:                     # one loop pass: its whole queue
+            seg = []
+            while i < n and int(events[i][0]) == EV_SEGMENT:
+                seg.append((int(events[i][2]), int(events[i][4])))
+                i += 1
+            cnt, base = {}, 0
+            for node, _ in seg:
+                x = parent[node]
+                while x != -1:
+                    if cnt.get(x, 0) == 0:
+                        base += tok[x]
+                    cnt[x] = cnt.get(x, 0) + 1
+                    x = parent[x]
+            alive, t = len(seg), 0
+            for node, ln in sorted(seg, key=lambda s: s[1]):
+                steps = ln - t                       # token steps t .. ln-1 with this many paths alive
+                if steps > 0:
+                    leaf_tok = alive * (steps * (t + 1 + ln)) // 2
+                    total += (base * steps + leaf_tok) * kv_tok
+                    rows += alive * steps
+                    t = ln
+                alive -= 1
+                x = parent[node]
+                while x != -1:
+                    cnt[x] -= 1
+                    if cnt[x] == 0:
+                        base -= tok[x]
+                    x = parent[x]
+            for node, ln in seg:
+                tok[node] = ln
+        else:
+            i += 1
+    return total + rows * q_row, rows
+
+
+def _clocks_start():
+    import torch
+    bus = getattr(torch.cuda.get_device_properties(0), "pci_bus_id", None)
+    sampler = ClockSampler(bus if isinstance(bus, str) else None)
+    sampler.start()
+    time.sleep(0.3)
+    return sampler
+
+
+def bench_rollout(args):
+    """Algorithm 1 at the paper's tree shape (64 prompts, w = 16, 14 x 512
+    segments, binary budget) with decode attention after every generated
+    token; one step = one whole rollout on the same forest."""
+    import torch
+
+    import paper_2508_17445_gb300 as tp
+    from paper_2508_17445_gb300 import build as lib_build
+    lib_build.build()
+    sh = dict(ROLLOUT_SHAPE)
+    if args.prompts is not None:
+        sh["n_prompts"] = args.prompts
+    import workloads
+    heads = workloads.Heads(28, 4, 128)
+    prompts = rollout_prompts(sh["n_prompts"], args.seed)
+    # pool for the largest possible trees: every query's budgeted segments
+    segs = sum(min(sh["init_branches"] * 2 ** j, sh["width"]) for j in range(sh["max_depth"]))
+    blocks = sum(-(-p // 32) for p in prompts) + sh["n_prompts"] * segs * (-(-sh["seg_tokens"] // 32))
+    forest = tp.Forest(heads.num_q_heads, heads.num_kv_heads, heads.head_dim, pool_blocks=blocks + 1024,
+                       device="cuda:0")
+
+    def params(step):
+        return tp.rollout_params(prompts, width=sh["width"], max_depth=sh["max_depth"], seg_tokens=sh["seg_tokens"],
+                                 init_branches=sh["init_branches"], p_eos=sh["p_eos"], p_boxed=sh["p_boxed"],
+                                 p_fail=sh["p_fail"], p_correct=sh["p_correct"], seed=args.seed * 1000 + step,
+                                 decode=1, decode_flags=args.flags)
+    for w in range(args.warmup):
+        forest.rollout(params(w))
+    forest.sync()
+    sampler = _clocks_start()
+    tp.tp_profile_start(forest.handle)
+    t0 = time.perf_counter()
+    stats, algo_bytes, rows = [], 0, 0
+    for k in range(args.steps):
+        ev, st = forest.rollout(params(args.warmup + k))
+        stats.append(st)
+        b, r = rollout_decode_bytes(ev, heads)
+        algo_bytes += b
+        rows += r
+    forest.sync()
+    wall = time.perf_counter() - t0
+    kt = tp.tp_profile_stop(forest.handle)
+    clocks = sampler.stop()
+    tokens = sum(st["tokens"] for st in stats)
+    trajs = sum(st["outputs"] for st in stats)
+    assert rows == sum(st["decode_rows"] for st in stats)
+    dec_ms = kt["decode"]["ms"]
+    peak, kind = peaks()
+    achieved = algo_bytes / (dec_ms / 1e3) / 1e9
+    launches = sum(v["launches"] for v in kt.values())
+    line = {
+        "metric": "tree rollout generated tokens/s (Algorithm 1, decode attention after every token)",
+        "value": tokens / wall, "unit": "tokens/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": wall / args.steps * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"rollout: {sh['n_prompts']} prompts (256..1024 tokens), w={sh['width']}, "
+                               f"{sh['max_depth']} x {sh['seg_tokens']}-token segments, b0={sh['init_branches']}, "
+                               f"binary budget, p_eos={sh['p_eos']:.2g}/token, p_boxed={sh['p_boxed']}, "
+                               f"p_fail={sh['p_fail']}; 28 q / 4 kv heads, head_dim 128",
+                   "decode_flags": args.flags, "l2": "decode reads up to GBs of path KV per call, no flush"},
+        "trajectories_per_s": trajs / wall,
+        "decode_calls_per_step": sum(st["decode_calls"] for st in stats) / args.steps,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                     "traffic": None, "kernel": "decode kernels inside the rollout",
+                     "algorithmic_bytes_per_step": algo_bytes / args.steps,
+                     "peak_source": f"{kind} hbm_gbs"},
+        "kernel_ms_per_step": {k: v["ms"] / args.steps for k, v in kt.items()},
+        "host_ms_per_step": (wall * 1e3 - sum(v["ms"] for v in kt.values())) / args.steps,
+        "e2e": {"value": tokens / wall, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0,
+                "note": "the rollout is host-driven end to end: value is already wall-clock through tp_rollout"},
+        "gpu_launches": int(launches), "clocks": clocks,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = rollout_cpu_baseline(prompts, sh, args, heads, min(args.cpu_seconds, 20.0))
+    print(json.dumps(line), flush=True)
+    forest.close()
+
+
+def rollout_cpu_baseline(prompts, sh, args, heads, budget_s):
+    """The oracle on the host cores: Algorithm 1's decisions for the same
+    rollout, plus fp64 path attention for a seeded sample of its decode rows,
+    scaled to tokens/s."""
+    import numpy as np
+
+    import oracle
+    import oracle.rollout as R
+    op = R.RolloutParams(prompt_tokens=prompts, width=sh["width"], max_depth=sh["max_depth"],
+                         seg_tokens=sh["seg_tokens"], init_branches=sh["init_branches"], p_eos=sh["p_eos"],
+                         p_boxed=sh["p_boxed"], p_fail=sh["p_fail"], p_correct=sh["p_correct"], seed=args.seed * 1000)
+    t0 = time.perf_counter()
+    res = R.rollout(op)
+    t_dec = time.perf_counter() - t0
+    segs = [e for e in res.events if e[0] == R.EV_SEGMENT]
+    tokens = sum(e[4] for e in segs)
+    rng = np.random.default_rng(0)
+    cores = os.cpu_count() or 1
+    done, t_att = 0, 0.0
+    while t_att < budget_s * 0.7 and done < 4096:
+        e = segs[int(rng.integers(0, len(segs)))]
+        node, t = int(e[2]), int(rng.integers(0, e[4]))
+        kb, vb = R.path_kv(res, op.seed, node, t + 1, heads.num_kv_heads, heads.head_dim)
+        qb = R.synth_rows(op.seed, R.TAG_Q, [node], [t], heads.num_q_heads, heads.head_dim)[0]
+        t1 = time.perf_counter()
+        oracle.path_attention(qb, kb, vb)
+        t_att += time.perf_counter() - t1
+        done += 1
+    per_row = t_att / done
+    total = t_dec + tokens * per_row
+    return {"value": tokens / total, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+            "sample": f"oracle Algorithm 1 over the whole rollout ({t_dec:.1f} s) + fp64 path attention for "
+                      f"{done} sampled (leaf, token) decode rows ({per_row * 1e3:.2f} ms each), scaled to its "
+                      f"{tokens} generated tokens; single thread"}
+
+
+def bench_prefill(args):
+    """Causal multi-query attention over tree paths: 64 prompts of 1024
+    tokens, each forked into 16 leaves holding a 512-token segment; one step
+    = one tp_prefill over every leaf's whole segment (524288 query tokens)."""
+    import torch
+
+    import paper_2508_17445_gb300 as tp
+    import workloads
+    from paper_2508_17445_gb300 import build as lib_build
+    lib_build.build()
+    n_prompts = args.prompts or 64
+    fan, plen, seg = 16, 1024, 512
+    script = workloads.segment_prefill(seed=args.seed, n_prompts=n_prompts, prompt_len=plen, fanout=fan, seg_len=seg)
+    h = script.heads
+    forest = tp.Forest(h.num_q_heads, h.num_kv_heads, h.head_dim, pool_blocks=script.upper_bound_blocks(32) + 64,
+                       device="cuda:0")
+    ids = forest.replay(script.ops, kv_fn=lambda i: script.kv(i, "cuda:0"))
+    nodes = [ids[x] for x in script.leaves]
+    counts = [seg] * len(nodes)
+    total = sum(counts)
+    g = torch.Generator(device="cpu").manual_seed(args.seed)
+    Q = torch.randn(total, h.num_q_heads, h.head_dim, generator=g).to(torch.bfloat16).to("cuda:0")
+    O = torch.empty_like(Q)
+    L = torch.empty(total, h.num_q_heads, dtype=torch.float32, device="cuda:0")
+    flops = 4 * h.head_dim * h.num_q_heads * len(nodes) * sum(plen + j + 1 for j in range(seg))
+    for _ in range(args.warmup):
+        tp.tp_prefill(forest.handle, nodes, counts, Q, O, L, args.flags)
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    sampler = _clocks_start()
+    tp.tp_profile_start(forest.handle)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.steps):
+        tp.tp_prefill(forest.handle, nodes, counts, Q, O, L, args.flags)
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / args.steps
+    kt = tp.tp_profile_stop(forest.handle)
+    clocks = sampler.stop()
+    forest.sync()
+    dec_ms = kt["decode"]["ms"] / max(kt["decode"]["launches"], 1)
+    peak, kind = peaks("bf16_tflops")
+    achieved = flops / (dec_ms / 1e3) / 1e12
+    # end to end: pinned host Q in, O and LSE back, every step
+    Qh, Oh = Q.cpu().pin_memory(), torch.empty(O.shape, dtype=O.dtype, pin_memory=True)
+    Lh = torch.empty(L.shape, dtype=L.dtype, pin_memory=True)
+    Qd = torch.empty_like(Q)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        Qd.copy_(Qh, non_blocking=True)
+        tp.tp_prefill(forest.handle, nodes, counts, Qd, O, L, args.flags)
+        Oh.copy_(O, non_blocking=True)
+        Lh.copy_(L, non_blocking=True)
+        stream.synchronize()
+    e2e_s = (time.perf_counter() - t0) / args.steps
+    line = {
+        "metric": "tree prefill query tokens/s (causal multi-query attention over root-to-node paths); "
+                  "TFLOP/s vs GB300 bf16 peak",
+        "value": total / (ms / 1e3), "unit": "query-tokens/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"segment_prefill: {n_prompts} prompts of {plen} tokens x {fan} leaves, each leaf's "
+                               f"{seg}-token segment as causal queries ({total} query tokens); 28 q / 4 kv heads, "
+                               f"head_dim 128",
+                   "flags": args.flags, "l2": "K/V re-read from L2 by the query blocks of a path; no flush"},
+        "tflops_call": flops / (ms / 1e3) / 1e12,
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": None, "kernel": "decode_tc_kernel (causal)",
+                     "algorithmic_flops_per_launch": flops, "launch_ms": dec_ms,
+                     "peak_source": f"{kind} bf16_tflops (burst)"},
+        "kernel_ms_per_step": {"attention": dec_ms, "merge": kt["merge"]["ms"] / max(kt["merge"]["launches"], 1)},
+        "e2e": {"value": total / e2e_s, "unit": "query-tokens/s", "h2d_bytes_per_step": Q.numel() * 2,
+                "d2h_bytes_per_step": O.numel() * 2 + L.numel() * 4},
+        "gpu_launches": int(kt["decode"]["launches"] + kt["merge"]["launches"]), "clocks": clocks,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = prefill_cpu_baseline(script, counts, Q, min(args.cpu_seconds, 20.0))
+    print(json.dumps(line), flush=True)
+    forest.close()
+
+
+def prefill_cpu_baseline(script, counts, Q, budget_s):
+    import numpy as np
+
+    import oracle
+    model = oracle.OracleForest(block_tokens=32, pool_blocks=script.upper_bound_blocks(32) + 64).replay(script)
+    cache = {}
+
+    def src(i):
+        if i not in cache:
+            k, v = script.kv(i, "cpu")
+            cache[i] = (oracle.bf16_bits(k), oracle.bf16_bits(v))
+        return cache[i]
+    total = sum(counts)
+    rng = np.random.default_rng(0)
+    cores = os.cpu_count() or 1
+    rows = sorted(set(int(x) for x in rng.integers(0, total, cores * 4)))
+    qc = Q.cpu()
+    model.prefill(list(script.leaves), counts, qc, src, indices=rows[:cores])   # materialise the paths
+    t0 = time.perf_counter()
+    model.prefill(list(script.leaves), counts, qc, src, indices=rows, threads=cores)
+    dt = time.perf_counter() - t0
+    n = len(rows)
+    while dt < budget_s / 4 and n < total:
+        more = sorted(set(int(x) for x in rng.integers(0, total, n)))
+        t0 = time.perf_counter()
+        model.prefill(list(script.leaves), counts, qc, src, indices=more, threads=cores)
+        dt += time.perf_counter() - t0
+        n += len(more)
+    return {"value": n / dt, "unit": "query-tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{n} seeded query rows of the same call, fp64 C oracle over each row's causal path prefix, "
+                      f"threads over rows; {dt:.1f} s"}
+
+
+def bench_advantage(args):
+    """Eq. tree_ae over the output trees of a paper-shaped rollout batch
+    (64 prompts, w = 16): one step = one tp_tree_advantage call."""
+    import numpy as np
+    import torch
+
+    import paper_2508_17445_gb300 as tp
+    from paper_2508_17445_gb300 import build as lib_build
+    lib_build.build()
+    sh = dict(ROLLOUT_SHAPE)
+    n_prompts = args.prompts or sh["n_prompts"]
+    prompts = rollout_prompts(n_prompts, args.seed)
+    dry = tp.Forest(28, 4, 128, pool_blocks=1 << 22, device=None)
+    ev, st = dry.rollout(tp.rollout_params(prompts, width=sh["width"], max_depth=sh["max_depth"],
+                                           seg_tokens=sh["seg_tokens"], init_branches=sh["init_branches"],
+                                           p_eos=sh["p_eos"], p_boxed=0.1, p_fail=sh["p_fail"], p_correct=0.5,
+                                           seed=args.seed))
+    n_nodes = int(st["nodes"])
+    parent = [dry.node_info(x)["parent"] for x in range(n_nodes)]
+    outs = ev[ev[:, 0] == 4]
+    leaves = outs[:, 2].astype(np.int32)
+    rewards = outs[:, 5].astype(np.float32)
+    dev = "cuda:0"
+    P = torch.tensor(parent, dtype=torch.int32, device=dev)
+    Lf = torch.tensor(leaves, dtype=torch.int32, device=dev)
+    Rw = torch.tensor(rewards, dtype=torch.float32, device=dev)
+    adv = torch.empty(len(leaves), dtype=torch.float32, device=dev)
+    stats = torch.zeros(4, dtype=torch.float64, device=dev)
+    ws = torch.empty(max(tp.tp_advantage_workspace_bytes(n_nodes, len(leaves)), 8), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        tp.tp_tree_advantage(P, Lf, Rw, adv, stats, ws, stream.cuda_stream)
+    torch.cuda.synchronize()
+    sampler = _clocks_start()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.steps):
+        tp.tp_tree_advantage(P, Lf, Rw, adv, stats, ws, stream.cuda_stream)
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / args.steps
+    clocks = sampler.stop()
+    depth = float(np.mean(outs[:, 3]))
+    algo = 4 * n_nodes + 12 * len(leaves) + 4 * int(len(leaves) * depth) * 2
+    peak, kind = peaks()
+    Lh, Rh = Lf.cpu().pin_memory(), Rw.cpu().pin_memory()
+    Ah = torch.empty(adv.shape, dtype=adv.dtype, pin_memory=True)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        Lf.copy_(Lh, non_blocking=True)
+        Rw.copy_(Rh, non_blocking=True)
+        tp.tp_tree_advantage(P, Lf, Rw, adv, stats, ws, stream.cuda_stream)
+        Ah.copy_(adv, non_blocking=True)
+        stream.synchronize()
+    e2e_s = (time.perf_counter() - t0) / args.steps
+    line = {
+        "metric": "tree advantage trajectories/s (Eq. tree_ae: sub-group means over the node table, "
+                  "mean pooling, global std)",
+        "value": len(leaves) / (ms / 1e3), "unit": "trajectories/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64 accumulation, f32 out", "data": "synthetic",
+        "config": {"workload": f"output trees of a {n_prompts}-prompt rollout batch (w=16, 14 x 512): "
+                               f"{len(leaves)} trajectories, {n_nodes} nodes, mean depth {depth:.1f}"},
+        "roofline": {"bound": "hbm", "achieved": algo / (ms / 1e3) / 1e9, "peak": peak, "unit": "GB/s",
+                     "frac": algo / (ms / 1e3) / 1e9 / peak, "traffic": None, "kernel": "advantage_kernel",
+                     "note": "one CTA; a few hundred KB per call: launch- and latency-bound, not bandwidth-bound",
+                     "peak_source": f"{kind} hbm_gbs"},
+        "e2e": {"value": len(leaves) / e2e_s, "unit": "trajectories/s", "h2d_bytes_per_step": 8 * len(leaves),
+                "d2h_bytes_per_step": 4 * len(leaves)},
+        "gpu_launches": args.steps, "clocks": clocks,
+    }
+    if not args.no_cpu_baseline:
+        import oracle.advantage as OA
+        t0 = time.perf_counter()
+        k = 0
+        while time.perf_counter() - t0 < min(args.cpu_seconds, 5.0) or k == 0:
+            OA.tree_advantage(parent, leaves.tolist(), rewards.astype(np.float64).tolist())
+            k += 1
+        dt = (time.perf_counter() - t0) / k
+        line["cpu_baseline"] = {"value": len(leaves) / dt, "unit": "trajectories/s", "cores": 1, "kind": "oracle",
+                                "sample": f"the whole call, {k} repetitions, fp64 Python loops, single thread"}
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------
 # the GPU arm
 # --------------------------------------------------------------------------
 def main():
@@ -300,6 +695,10 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.workload in ("rollout", "prefill", "advantage"):
+        if rank == 0:     # single-GPU measurements of the other paths; other ranks have no work
+            {"rollout": bench_rollout, "prefill": bench_prefill, "advantage": bench_advantage}[args.workload](args)
+        return
     if args.impl == "reference":
         run_reference(args, rank, world)
         return

@@ -26,7 +26,7 @@ __all__ = [
     "tp_debug_schedule", "tp_decode_noalloc", "tp_append_tokens", "tp_synth_tokens", "tp_branch_assign",
     "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "tp_prefill", "tp_debug_prefill_schedule", "TpRolloutParams", "TpRolloutStats",
     "TpRolloutProbe", "rollout_params", "TP_BRANCH_EVEN", "TP_BRANCH_LOGP_HIGH", "TP_BRANCH_LOGP_LOW",
-    "EVENT_NAMES", "TP_SEG_EOS", "TP_SEG_BOXED", "TP_SEG_FAILED", "TP_SEG_MAX_DEPTH", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE", "TP_DECODE_TCGEN05", "TP_DECODE_ALL_TCGEN05", "TP_PREFILL_MMA_SYNC",
+    "EVENT_NAMES", "TP_SEG_EOS", "TP_SEG_BOXED", "TP_SEG_FAILED", "TP_SEG_MAX_DEPTH", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE", "TP_DECODE_TCGEN05", "TP_DECODE_ALL_TCGEN05", "TP_MMA_SYNC",
     "EXPORTED_SYMBOLS",
 ]
 
@@ -39,7 +39,7 @@ TP_DECODE_CUDA_CORE_SMALL = 2
 TP_DECODE_NO_CACHE = 4
 TP_DECODE_TCGEN05 = 8
 TP_DECODE_ALL_TCGEN05 = 16
-TP_PREFILL_MMA_SYNC = 32
+TP_MMA_SYNC = 32
 
 TP_BRANCH_EVEN = 0
 TP_BRANCH_LOGP_HIGH = 1

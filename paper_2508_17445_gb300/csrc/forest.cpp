@@ -132,8 +132,10 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     const int32_t hq = t->cfg.num_q_heads, hkv = t->cfg.num_kv_heads, g = hq / hkv;
     const bool share = !(flags & TP_DECODE_NO_SHARE);
     const bool cuda_core_small = (flags & TP_DECODE_CUDA_CORE_SMALL) != 0;
-    const bool all_tc = (flags & TP_DECODE_ALL_TCGEN05) != 0;
-    const bool use_tc = all_tc || (flags & TP_DECODE_TCGEN05) != 0;
+    // tcgen05 for every unit of more than one 16-row MMA tile unless
+    // TP_MMA_SYNC; TP_DECODE_TCGEN05 alone keeps it to long, tall chunks
+    const bool use_tc = (flags & TP_MMA_SYNC) == 0;
+    const bool all_tc = use_tc && !((flags & TP_DECODE_TCGEN05) && !(flags & TP_DECODE_ALL_TCGEN05));
     for (int32_t i = 0; i < n; ++i) {
         tp_status st = check_live(t, leaves[i], true);
         if (st != TP_OK) return st;
@@ -393,7 +395,7 @@ tp_status build_prefill_schedule(tp_tree* t, const tp_node* nodes, const int32_t
     }
     if (n_q >= (int64_t)1 << 28) return fail(t, TP_ERR_INVALID_ARG, "too many query tokens in one call");
     SchedScratch& X = t->scratch;
-    const bool use_tc = !(flags & TP_PREFILL_MMA_SYNC);  // tcgen05 unless asked otherwise (measured faster)
+    const bool use_tc = !(flags & TP_MMA_SYNC);  // tcgen05 unless asked otherwise (measured faster)
     const int32_t occ_per_block = (use_tc ? kTcRowsPerUnit : kTensorRowsPerUnit) / g;  // whole GQA groups
     // path tiles of every listed node, with each tile's path position
     X.tiles.clear();

@@ -29,11 +29,10 @@ constexpr int32_t kSchedMagic = 0x54505344;
 constexpr int kTensorMinRows = 16;
 // Query rows per mma.sync unit (4 warps x one 16-row MMA tile each).
 constexpr int kTensorRowsPerUnit = 64;
-// tcgen05 units (128 rows, MMA M) are opt-in: TP_DECODE_TCGEN05 sends chunks
-// of at least kTcMinRows stacked rows per kv head and kTcMinTiles blocks,
-// TP_DECODE_ALL_TCGEN05 every unit of more than one 16-row MMA tile. By
-// default every unit runs on mma.sync, which measured faster on GB300: the
-// tcgen05 pipeline pays a longer start and drain per unit.
+// tcgen05 units (128 rows, MMA M): by default every unit of more than one
+// 16-row MMA tile (kTcAnyRows); TP_DECODE_TCGEN05 alone keeps tcgen05 to
+// chunks of at least kTcMinRows stacked rows per kv head and kTcMinTiles
+// blocks; TP_MMA_SYNC runs all stacked rows on mma.sync in 64-row units.
 constexpr int kTcMinRows = 64;
 constexpr int kTcMinTiles = 32;
 constexpr int kTcAnyRows = 17;

@@ -101,7 +101,7 @@ def run_and_compare(script, flags=0, sample=None, leaves=None, q=None):
     return O, LSE, err
 
 
-FLAG_SETS = [0, tp.TP_DECODE_CUDA_CORE_SMALL, tp.TP_DECODE_NO_SHARE, tp.TP_DECODE_ALL_TCGEN05]
+FLAG_SETS = [0, tp.TP_DECODE_CUDA_CORE_SMALL, tp.TP_DECODE_NO_SHARE, tp.TP_MMA_SYNC]
 
 
 # --------------------------------------------------------------------------
@@ -132,7 +132,7 @@ def test_random_divergence_reduced(flags):
     run_and_compare(workloads.random_divergence(seed=2, n_prompts=3, depth=5), flags)
 
 
-@pytest.mark.parametrize("flags", [0, tp.TP_DECODE_NO_SHARE, tp.TP_DECODE_TCGEN05, tp.TP_DECODE_ALL_TCGEN05])
+@pytest.mark.parametrize("flags", [0, tp.TP_DECODE_NO_SHARE, tp.TP_DECODE_TCGEN05, tp.TP_MMA_SYNC])
 def test_wide_prefix_one_prompt(flags):
     # root shared by 64 leaves x 8 heads = 512 rows: 8 tensor units per chunk
     run_and_compare(workloads.wide_prefix(seed=3, n_prompts=1), flags)
@@ -315,7 +315,7 @@ def test_full_size_sampled(name, k):
     rows = _sample(len(leaf_ids), k, seed=len(name))
     src = _kv_source(s)
     o_ref, lse_ref, a_ref = oracle_outputs(model, s.leaves, Q.cpu(), src, rows)
-    for flags in (0, tp.TP_DECODE_CUDA_CORE_SMALL, tp.TP_DECODE_ALL_TCGEN05, tp.TP_DECODE_TCGEN05):
+    for flags in (0, tp.TP_DECODE_CUDA_CORE_SMALL, tp.TP_MMA_SYNC, tp.TP_DECODE_TCGEN05):
         O, LSE = f.decode(leaf_ids, Q, flags=flags)
         f.sync()
         check(O, LSE, o_ref, lse_ref, a_ref, rows=rows)

@@ -67,7 +67,7 @@ def run_prefill(script, nodes_sid, counts, rows=None, seed=0, flags=0):
     return O, LSE
 
 
-FLAGS = [0, tp.TP_PREFILL_MMA_SYNC]
+FLAGS = [0, tp.TP_MMA_SYNC]
 
 
 @pytest.mark.parametrize("flags", FLAGS)

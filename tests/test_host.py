@@ -260,6 +260,7 @@ def check_schedule(f, ids, model, script, leaves_sid, flags=0):
     leaves = [ids[x] for x in leaves_sid]
     S = tp.tp_debug_schedule(f.handle, leaves, flags)
     assert S["group"] == g
+    all_tc = not flags & tp.TP_MMA_SYNC and not (flags & tp.TP_DECODE_TCGEN05 and not flags & tp.TP_DECODE_ALL_TCGEN05)
     covered = collections.defaultdict(list)
     slots_of = collections.defaultdict(set)
     chunk_reads = collections.Counter()
@@ -268,17 +269,17 @@ def check_schedule(f, ids, model, script, leaves_sid, flags=0):
         assert 0 <= kvh < heads.num_kv_heads
         if kind == 0:                      # CUDA-core: one leaf group, < 16 rows
             assert nrows < 16 and flags & tp.TP_DECODE_CUDA_CORE_SMALL
-        elif kind == 1:                    # mma.sync: 64-row blocks (<= 16 rows with all-tcgen05)
-            if flags & tp.TP_DECODE_ALL_TCGEN05:
+        elif kind == 1:                    # mma.sync: one 16-row tile (all-tcgen05), else 64-row blocks
+            if all_tc:
                 assert row0 == 0 and 1 <= nrows <= 16
             else:
                 assert 1 <= nrows <= 64
             if flags & tp.TP_DECODE_CUDA_CORE_SMALL:
                 assert nrows >= 16 or row0 > 0
-        else:                              # tcgen05 (opt-in): stacked rows in 128-row blocks
-            assert kind == 2 and flags & (tp.TP_DECODE_TCGEN05 | tp.TP_DECODE_ALL_TCGEN05)
+        else:                              # tcgen05: stacked rows in 128-row blocks
+            assert kind == 2 and not flags & tp.TP_MMA_SYNC
             assert 1 <= nrows <= 128
-            if flags & tp.TP_DECODE_ALL_TCGEN05:
+            if all_tc:
                 assert row0 > 0 or nrows >= 17
             else:
                 assert nt >= 32 and (row0 > 0 or nrows >= 64)
@@ -307,7 +308,7 @@ def check_schedule(f, ids, model, script, leaves_sid, flags=0):
 
 @pytest.mark.parametrize("seed", range(6))
 @pytest.mark.parametrize("flags", [0, tp.TP_DECODE_NO_SHARE, tp.TP_DECODE_CUDA_CORE_SMALL, tp.TP_DECODE_TCGEN05,
-                                   tp.TP_DECODE_ALL_TCGEN05])
+                                   tp.TP_DECODE_ALL_TCGEN05, tp.TP_MMA_SYNC])
 def test_schedule_covers_every_path_token_once(seed, flags):
     s = workloads.random_tree(seed=seed, n_prompts=3, max_depth=5, prompt_range=(1, 300), seg_range=(1, 150),
                               heads=workloads.Heads(8, 2, 64))

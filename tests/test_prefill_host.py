@@ -24,7 +24,7 @@ def check_prefill_coverage(f, model, ids, nodes_sid, counts, flags=0):
     nodes = [ids[x] for x in nodes_sid]
     d = tp.tp_debug_prefill_schedule(f.handle, nodes, counts, flags)
     units, tiles = d["units"], d["tiles"]
-    tc = not (flags & tp.TP_PREFILL_MMA_SYNC)
+    tc = not (flags & tp.TP_MMA_SYNC)
     assert len(d["vis"]) == sum(counts) and np.array_equal(d["occ"], np.arange(sum(counts)))
     assert np.all(units[:, 7] == (2 if tc else 1)) and np.all(units[:, 4] % g == 0)
     assert np.all(units[:, 4] <= (128 if tc else 64))
@@ -73,7 +73,7 @@ def check_prefill_coverage(f, model, ids, nodes_sid, counts, flags=0):
         r += mq
 
 
-@pytest.mark.parametrize("flags", [0, tp.TP_PREFILL_MMA_SYNC])
+@pytest.mark.parametrize("flags", [0, tp.TP_MMA_SYNC])
 @pytest.mark.parametrize("seed", range(8))
 def test_prefill_schedule_covers_each_visible_token_once(seed, flags):
     s = workloads.random_tree(seed=seed, n_prompts=3, max_depth=4, heads=workloads.Heads(8, 2, 64))
@@ -94,8 +94,8 @@ def test_prefill_schedule_long_paths_are_chunked_and_clipped():
     model = oracle.OracleForest(block_tokens=32).replay(s)
     leaf = s.leaves[0]
     check_prefill_coverage(f, model, ids, [leaf], [600])
-    check_prefill_coverage(f, model, ids, [leaf], [600], tp.TP_PREFILL_MMA_SYNC)
-    d = tp.tp_debug_prefill_schedule(f.handle, [ids[leaf]], [600], tp.TP_PREFILL_MMA_SYNC)
+    check_prefill_coverage(f, model, ids, [leaf], [600], tp.TP_MMA_SYNC)
+    d = tp.tp_debug_prefill_schedule(f.handle, [ids[leaf]], [600], tp.TP_MMA_SYNC)
     assert d["units"][:, 1].max() <= 128
     first_block = d["units"][d["units"][:, 2] == 0]
     last_block = d["units"][d["units"][:, 2] == d["units"][:, 2].max()]
