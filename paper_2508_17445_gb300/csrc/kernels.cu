@@ -1567,15 +1567,26 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
             tmem_ld32_nowait(s_addr, r[0]);
             tmem_ld32_nowait(s_addr + 32, r[1]);
             tmem_wait_ld();
-            // row max over the tokens the row may see
+            // row max over the tokens the row may see, on the raw scores (the
+            // scale is positive); a stage every row of the warp sees whole
+            // takes the unmasked path
+            const bool whole = __all_sync(0xffffffffu, lim0 == 32 && lim1 == 32);
             float mx = -INFINITY;
+            if (whole) {
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int lim = h ? lim1 : lim0;
+                for (int h = 0; h < 2; ++h)
 #pragma unroll
-                for (int t = 0; t < 32; ++t)
-                    if (t < lim) mx = fmaxf(mx, __uint_as_float(r[h][t]) * a.qk_scale_log2);
+                    for (int t = 0; t < 32; ++t) mx = fmaxf(mx, __uint_as_float(r[h][t]));
+            } else {
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int lim = h ? lim1 : lim0;
+#pragma unroll
+                    for (int t = 0; t < 32; ++t)
+                        if (t < lim) mx = fmaxf(mx, __uint_as_float(r[h][t]));
+                }
             }
+            mx *= a.qk_scale_log2;
             const float m_new = fmaxf(m_used, mx);
             const bool need = m_new > m_used + kRescaleLog2;
             if (__any_sync(0xffffffffu, need)) {
@@ -1597,19 +1608,31 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
                     m_used = m_new;
                 }
             }
-            // P = exp2(s - m_used) as bf16 pairs over the S columns
+            // P = exp2(s * scale - m_used) as bf16 pairs over the S columns
             uint32_t pw[32];
             float sum = 0.f;
+            const float sc = a.qk_scale_log2, neg_m = -m_used;
+            if (whole) {
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int lim = h ? lim1 : lim0;
+                for (int h = 0; h < 2; ++h)
 #pragma unroll
-                for (int t = 0; t < 32; t += 2) {
-                    const float p0 = t < lim ? fast_exp2(__uint_as_float(r[h][t]) * a.qk_scale_log2 - m_used) : 0.f;
-                    const float p1 =
-                        t + 1 < lim ? fast_exp2(__uint_as_float(r[h][t + 1]) * a.qk_scale_log2 - m_used) : 0.f;
-                    sum += p0 + p1;
-                    pw[h * 16 + t / 2] = pack_bf16(p0, p1);
+                    for (int t = 0; t < 32; t += 2) {
+                        const float p0 = fast_exp2(fmaf(__uint_as_float(r[h][t]), sc, neg_m));
+                        const float p1 = fast_exp2(fmaf(__uint_as_float(r[h][t + 1]), sc, neg_m));
+                        sum += p0 + p1;
+                        pw[h * 16 + t / 2] = pack_bf16(p0, p1);
+                    }
+            } else {
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int lim = h ? lim1 : lim0;
+#pragma unroll
+                    for (int t = 0; t < 32; t += 2) {
+                        const float p0 = t < lim ? fast_exp2(fmaf(__uint_as_float(r[h][t]), sc, neg_m)) : 0.f;
+                        const float p1 = t + 1 < lim ? fast_exp2(fmaf(__uint_as_float(r[h][t + 1]), sc, neg_m)) : 0.f;
+                        sum += p0 + p1;
+                        pw[h * 16 + t / 2] = pack_bf16(p0, p1);
+                    }
                 }
             }
             l += sum;
