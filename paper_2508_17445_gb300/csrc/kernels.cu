@@ -111,6 +111,12 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
         : "memory");
 }
 
+// 16-byte global -> shared copy that bypasses registers (cp.async)
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
 __device__ __forceinline__ void fence_proxy_async() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -1309,28 +1315,29 @@ __device__ void tc_fetch(const DecodeArgs& a, CtlTc& c, uint8_t* qbuf) {
         // the previous unit's Q.K^T MMAs have read the buffer
         if (!mbar_wait(smem_u32(&c.qempty), (k & 1) ^ 1)) note_timeout(a, c, 2);
         constexpr int CH = HD / 8;  // 16-byte chunks per row
-        constexpr int BATCH = 16;   // loads in flight per lane
         const int g = a.group;
-        for (int r = lane; r < n_rows; r += 32) {  // row pointers: one round trip
-            const int item_row = row0 + r;
-            c.qrow[r] = ((int64_t)a.occ[occ_off + item_row / g] * a.hq + kvh * g + item_row % g) * HD;
+        // prefill schedules list query rows in order (occurrence = query
+        // index), so their row addresses need no lookup
+        const bool in_order = a.vis != nullptr;
+        if (!in_order) {
+            for (int r = lane; r < n_rows; r += 32) {  // row pointers: one round trip
+                const int item_row = row0 + r;
+                c.qrow[r] = ((int64_t)a.occ[occ_off + item_row / g] * a.hq + kvh * g + item_row % g) * HD;
+            }
+            __syncwarp();
         }
-        __syncwarp();
+        // 16-byte async copies straight into the swizzled layout: every
+        // chunk of the tile in flight at once, no registers
         const int total = n_rows * CH;
-        for (int base = 0; base < total; base += 32 * BATCH) {
-            uint4 v[BATCH];
-#pragma unroll
-            for (int b = 0; b < BATCH; ++b) {
-                const int idx = base + b * 32 + lane;
-                if (idx < total) v[b] = *reinterpret_cast<const uint4*>(a.q + c.qrow[idx / CH] + (idx % CH) * 8);
-            }
-#pragma unroll
-            for (int b = 0; b < BATCH; ++b) {
-                const int idx = base + b * 32 + lane;
-                if (idx < total) *reinterpret_cast<uint4*>(qbuf + kv_off<kTcRows>(idx / CH, idx % CH)) = v[b];
-            }
+        for (int idx = lane; idx < total; idx += 32) {
+            const int r = idx / CH, ch = idx % CH;
+            const int item_row = row0 + r;
+            const int64_t off = in_order ? ((int64_t)(occ_off + item_row / g) * a.hq + kvh * g + item_row % g) * HD
+                                         : c.qrow[r];
+            cp_async16(smem_u32(qbuf + kv_off<kTcRows>(r, ch)), a.q + off + ch * 8);
         }
-        fence_proxy_async();  // generic stores -> visible to the tensor core
+        cp_async_wait_all();
+        fence_proxy_async();  // the copies -> visible to the tensor core
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&c.qfull));
     }
