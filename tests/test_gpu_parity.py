@@ -166,6 +166,18 @@ def test_long_shared_prompt_is_chunked(flags):
     run_and_compare(s, flags)
 
 
+@pytest.mark.parametrize("flags", FLAG_SETS)
+def test_more_slots_than_one_merge_chunk(flags):
+    # a 12000-token path at head_dim 128 is cut into more than 32 chunks: the
+    # merge folds the slots 32 at a time and rescales across the chunks
+    s = workloads.single_path(seed=12, lengths=(12000,), heads=workloads.Heads(8, 1, 128))
+    f, ids = build_forest(s)
+    sched = tp.tp_debug_schedule(f.handle, [ids[x] for x in s.leaves], flags)
+    f.close()
+    assert max(np.diff(sched["merge_off"])) > 32
+    run_and_compare(s, flags)
+
+
 def test_repeated_leaf_gives_bitwise_identical_rows():
     s = workloads.random_tree(seed=5, heads=workloads.Heads(28, 4, 128), n_prompts=2)
     f, ids = build_forest(s)
