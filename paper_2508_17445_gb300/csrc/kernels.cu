@@ -1187,7 +1187,6 @@ struct CtlTc {
     int unit[2];
     int desc[2][kUnitWords + 1];  // + path position of the unit's first token (prefill)
     int tiles[2][kMaxUnitTiles];
-    int64_t qrow[kTcRows];    // element offset in Q of each row being staged
     uint32_t tmem;
     int abort;
 };
@@ -1316,25 +1315,32 @@ __device__ void tc_fetch(const DecodeArgs& a, CtlTc& c, uint8_t* qbuf) {
         if (!mbar_wait(smem_u32(&c.qempty), (k & 1) ^ 1)) note_timeout(a, c, 2);
         constexpr int CH = HD / 8;  // 16-byte chunks per row
         const int g = a.group;
-        // prefill schedules list query rows in order (occurrence = query
-        // index), so their row addresses need no lookup
+        // lane = query row (rows lane, lane + 32, ...): its source row is
+        // found once -- prefill schedules list query rows in order
+        // (occurrence = query index), decode looks the occurrence up, all
+        // lookups in flight together -- then its CH chunks go out as 16-byte
+        // async copies straight into the swizzled layout, offsets known at
+        // compile time, every copy of the tile in flight at once
+        constexpr int kRowsPerLane = kTcRows / 32;
         const bool in_order = a.vis != nullptr;
-        if (!in_order) {
-            for (int r = lane; r < n_rows; r += 32) {  // row pointers: one round trip
-                const int item_row = row0 + r;
-                c.qrow[r] = ((int64_t)a.occ[occ_off + item_row / g] * a.hq + kvh * g + item_row % g) * HD;
-            }
-            __syncwarp();
+        int64_t src_off[kRowsPerLane];
+#pragma unroll
+        for (int i = 0; i < kRowsPerLane; ++i) {
+            const int r = lane + 32 * i;
+            const int item_row = row0 + r, p = item_row / g, hh = item_row - p * g;
+            const int occ = r >= n_rows ? 0 : in_order ? occ_off + p : a.occ[occ_off + p];
+            src_off[i] = ((int64_t)occ * a.hq + kvh * g + hh) * HD;
         }
-        // 16-byte async copies straight into the swizzled layout: every
-        // chunk of the tile in flight at once, no registers
-        const int total = n_rows * CH;
-        for (int idx = lane; idx < total; idx += 32) {
-            const int r = idx / CH, ch = idx % CH;
-            const int item_row = row0 + r;
-            const int64_t off = in_order ? ((int64_t)(occ_off + item_row / g) * a.hq + kvh * g + item_row % g) * HD
-                                         : c.qrow[r];
-            cp_async16(smem_u32(qbuf + kv_off<kTcRows>(r, ch)), a.q + off + ch * 8);
+        const uint32_t q_base = smem_u32(qbuf);
+#pragma unroll
+        for (int i = 0; i < kRowsPerLane; ++i) {
+            const int r = lane + 32 * i;
+            if (r >= n_rows) break;
+            const uint16_t* src = a.q + src_off[i];
+            const uint32_t dst = q_base + r * 128, x = r & 7;
+#pragma unroll
+            for (int ch = 0; ch < CH; ++ch)
+                cp_async16(dst + (ch >> 3) * (kTcRows * 128) + (((ch & 7) ^ x) << 4), src + ch * 8);
         }
         cp_async_wait_all();
         fence_proxy_async();  // the copies -> visible to the tensor core
