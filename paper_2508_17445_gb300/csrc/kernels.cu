@@ -146,6 +146,34 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// max of three (one instruction on sm_100 and later)
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
+// Packed fp32 pairs (sm_100 and later): one instruction, two lanes, each
+// rounded exactly like its scalar counterpart.
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+
 // bf16 pair in a 32-bit word -> two fp32 (exact: bf16 is the top half of fp32)
 __device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
@@ -1585,11 +1613,16 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
             // takes the unmasked path
             const bool whole = __all_sync(0xffffffffu, lim0 == 32 && lim1 == 32);
             float mx = -INFINITY;
-            if (whole) {
+            if (whole) {  // four independent chains of three-input maxima
+                float m0 = -INFINITY, m1 = -INFINITY, m2 = -INFINITY, m3 = -INFINITY;
 #pragma unroll
-                for (int h = 0; h < 2; ++h)
-#pragma unroll
-                    for (int t = 0; t < 32; ++t) mx = fmaxf(mx, __uint_as_float(r[h][t]));
+                for (int t = 0; t < 32; t += 4) {
+                    m0 = fmax3(m0, __uint_as_float(r[0][t]), __uint_as_float(r[0][t + 1]));
+                    m1 = fmax3(m1, __uint_as_float(r[0][t + 2]), __uint_as_float(r[0][t + 3]));
+                    m2 = fmax3(m2, __uint_as_float(r[1][t]), __uint_as_float(r[1][t + 1]));
+                    m3 = fmax3(m3, __uint_as_float(r[1][t + 2]), __uint_as_float(r[1][t + 3]));
+                }
+                mx = fmaxf(fmax3(m0, m1, m2), m3);
             } else {
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
@@ -1625,16 +1658,24 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
             uint32_t pw[32];
             float sum = 0.f;
             const float sc = a.qk_scale_log2, neg_m = -m_used;
-            if (whole) {
+            if (whole) {  // scale and shift two scores per instruction; two pair sums
+                const uint64_t sc2 = f2_pack(sc, sc), nm2 = f2_pack(neg_m, neg_m);
+                uint64_t acc[2] = {0, 0};
 #pragma unroll
                 for (int h = 0; h < 2; ++h)
 #pragma unroll
                     for (int t = 0; t < 32; t += 2) {
-                        const float p0 = fast_exp2(fmaf(__uint_as_float(r[h][t]), sc, neg_m));
-                        const float p1 = fast_exp2(fmaf(__uint_as_float(r[h][t + 1]), sc, neg_m));
-                        sum += p0 + p1;
+                        float x0, x1;
+                        f2_unpack(f2_fma(f2_pack(__uint_as_float(r[h][t]), __uint_as_float(r[h][t + 1])), sc2, nm2),
+                                  x0, x1);
+                        const float p0 = fast_exp2(x0), p1 = fast_exp2(x1);
+                        acc[(t >> 1) & 1] = f2_add(acc[(t >> 1) & 1], f2_pack(p0, p1));
                         pw[h * 16 + t / 2] = pack_bf16(p0, p1);
                     }
+                float s0, s1, s2, s3;
+                f2_unpack(acc[0], s0, s1);
+                f2_unpack(acc[1], s2, s3);
+                sum = (s0 + s2) + (s1 + s3);
             } else {
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
