@@ -1198,19 +1198,24 @@ struct TcSmem {
     static constexpr int kBytes = kRingBytes + kQBytes + 1024;  // + slack to align to 1024
 };
 
+static_assert(kStages == 2, "the S buffers and the ring slots share their index");
+
 struct CtlTc {
+    // Each tcgen05.commit costs the issuing thread about as long as an MMA,
+    // so one commit serves every waiter of the same completion: s_full[s]
+    // also frees ring slot s's K half (the S buffer and the ring slot of a
+    // stage share its index, kStages = 2), and vempty[s] also tells the
+    // softmax that the P.V of the stage in slot s has finished.
     uint64_t kfull[kStages];   // K half of the stage landed (streamer + TMA bytes)
-    uint64_t kempty[kStages];  // K half read by Q.K^T (issuer's commit)
     uint64_t vfull[kStages];   // V half landed
     uint64_t vempty[kStages];  // V half read by P.V (issuer's commit)
     uint64_t ufull[2], uempty[2];
     uint64_t qfull;           // query rows staged (fetcher)
     uint64_t qempty;          // the unit's last Q.K^T done (issuer's commit)
-    uint64_t s_full[2];       // S buffer holds scores (issuer's commit)
+    uint64_t s_full[2];       // S buffer holds scores, K half read (issuer's commit)
     uint64_t p_full[2];       // S buffer holds P (one arrival per consumer warp)
     uint64_t o_full;          // the unit's last P.V done (issuer's commit)
     uint64_t o_free;          // the epilogue has read O (one arrival per consumer warp)
-    uint64_t pv_done;         // a P.V finished (issuer's commit; rescale waits)
     int valid[kStages][2];
     int unit[2];
     int desc[2][kUnitWords + 1];  // + path position of the unit's first token (prefill)
@@ -1424,7 +1429,7 @@ __device__ void tc_stream(const DecodeArgs& a, CtlTc& c, uint8_t* ring) {
         uint32_t spins = 0;
         while (vj < n_pairs) {
             bool progress = false;
-            if (kj < n_pairs && mbar_test(smem_u32(&c.kempty[ks]), kph ^ 1)) {
+            if (kj < n_pairs && mbar_test(smem_u32(&c.s_full[ks]), kph ^ 1)) {  // K slot read by Q.K^T
                 const int32_t w[2] = {tw[2 * kj], 2 * kj + 1 < n_tiles ? tw[2 * kj + 1] : -1};
                 fence_proxy_async();
                 issue_half<HD>(a, kvh, 0, ring + ks * TcSmem<HD>::kStageBytes, w, smem_u32(&c.kfull[ks]));
@@ -1506,8 +1511,7 @@ __device__ void tc_issue(const DecodeArgs& a, CtlTc& c, const uint8_t* ring, con
                     const uint32_t qoff = (ks >> 2) * (kTcRows * 128) + (ks & 3) * 32;
                     mma_ss(d, smem_desc(q_addr + qoff, 16, 1024), smem_desc(kb + off, 16, 1024), kIdescS, ks > 0);
                 }
-                tc_commit(smem_u32(&c.s_full[g_stage & 1]));
-                tc_commit(smem_u32(&c.kempty[s_stage]));
+                tc_commit(smem_u32(&c.s_full[g_stage & 1]));  // = ring slot s_stage
                 if (++s_stage == kStages) {
                     s_stage = 0;
                     s_phase ^= 1;
@@ -1535,7 +1539,6 @@ __device__ void tc_issue(const DecodeArgs& a, CtlTc& c, const uint8_t* ring, con
                            smem_desc(vb + kk * 2048, kStageTokens * 128, 1024), kIdescPV,
                            (next_pv > 0 || kk > 0) ? 1u : 0u);
                 tc_commit(smem_u32(&c.vempty[v_stage]));
-                tc_commit(smem_u32(&c.pv_done));
                 if (next_pv + 1 == n_pairs) tc_commit(smem_u32(&c.o_full));
                 if (++v_stage == kStages) {
                     v_stage = 0;
@@ -1638,7 +1641,8 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
             if (__any_sync(0xffffffffu, need)) {
                 const float alpha = need ? fast_exp2(m_used - m_new) : 1.f;
                 if (j > 0) {  // O holds earlier stages: wait for the last P.V, then scale it
-                    if (!mbar_wait(smem_u32(&c.pv_done), (g_stage - 1) & 1)) note_timeout(a, c, 1);
+                    const uint32_t prev = g_stage - 1;  // its P.V used ring slot prev & 1
+                    if (!mbar_wait(smem_u32(&c.vempty[prev & 1]), (prev >> 1) & 1)) note_timeout(a, c, 1);
                     tc_fence_after();
 #pragma unroll 1
                     for (int cc = 0; cc < HD / 32; ++cc) {
@@ -1770,7 +1774,6 @@ __global__ void __launch_bounds__(kTcThreads, 2) decode_tc_kernel(const DecodeAr
     if (tid == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(smem_u32(&ctl.kfull[s]), 1);
-            mbar_init(smem_u32(&ctl.kempty[s]), 1);
             mbar_init(smem_u32(&ctl.vfull[s]), 1);
             mbar_init(smem_u32(&ctl.vempty[s]), 1);
         }
@@ -1784,7 +1787,6 @@ __global__ void __launch_bounds__(kTcThreads, 2) decode_tc_kernel(const DecodeAr
         mbar_init(smem_u32(&ctl.qempty), 1);
         mbar_init(smem_u32(&ctl.o_full), 1);
         mbar_init(smem_u32(&ctl.o_free), kTcConsumerWarps);
-        mbar_init(smem_u32(&ctl.pv_done), 1);
         ctl.abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
