@@ -146,6 +146,13 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// 32-byte global store (sm_100 and later); dst must be 32-byte aligned
+__device__ __forceinline__ void st_global_v8(void* dst, const uint32_t* w) {
+    asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(dst), "r"(w[0]), "r"(w[1]),
+                 "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                 : "memory");
+}
+
 // max of three (one instruction on sm_100 and later)
 __device__ __forceinline__ float fmax3(float a, float b, float c) {
     float r;
@@ -1729,24 +1736,42 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
             }
         }
         const float inv = 1.f / l;
+        // 32-byte stores (a full sector per lane) where the rows allow them:
+        // the partial buffer always, the caller's O when its base is 32-byte
+        // aligned (rows are multiples of 256 bytes, so the base decides)
+        const bool wide = !final_out || (reinterpret_cast<uintptr_t>(a.out) & 31) == 0;
 #pragma unroll 1
-        for (int cc = 0; cc < HD / 32; ++cc) {
-            uint32_t ov[32];
-            tmem_ld32(o_addr + cc * 32, ov);
-            if (live && final_out) {
+        for (int cc = 0; cc < HD / 32; cc += 2) {  // two 32-column loads in flight
+            uint32_t ov[2][32];
+            __syncwarp();  // the loads are warp-collective
+            tmem_ld32_nowait(o_addr + cc * 32, ov[0]);
+            tmem_ld32_nowait(o_addr + cc * 32 + 32, ov[1]);
+            tmem_wait_ld();
 #pragma unroll
-                for (int t = 0; t < 32; t += 8)
-                    *reinterpret_cast<uint4*>(dst16 + cc * 32 + t) =
-                        make_uint4(pack_bf16(__uint_as_float(ov[t]) * inv, __uint_as_float(ov[t + 1]) * inv),
-                                   pack_bf16(__uint_as_float(ov[t + 2]) * inv, __uint_as_float(ov[t + 3]) * inv),
-                                   pack_bf16(__uint_as_float(ov[t + 4]) * inv, __uint_as_float(ov[t + 5]) * inv),
-                                   pack_bf16(__uint_as_float(ov[t + 6]) * inv, __uint_as_float(ov[t + 7]) * inv));
-            } else if (live) {
+            for (int h = 0; h < 2 && live; ++h) {
+                const int c0 = (cc + h) * 32;
+                if (final_out) {
+                    uint32_t w[16];
 #pragma unroll
-                for (int t = 0; t < 32; t += 4)
-                    *reinterpret_cast<float4*>(dst + cc * 32 + t) =
-                        make_float4(__uint_as_float(ov[t]) * inv, __uint_as_float(ov[t + 1]) * inv,
-                                    __uint_as_float(ov[t + 2]) * inv, __uint_as_float(ov[t + 3]) * inv);
+                    for (int t = 0; t < 16; ++t)
+                        w[t] = pack_bf16(__uint_as_float(ov[h][2 * t]) * inv, __uint_as_float(ov[h][2 * t + 1]) * inv);
+                    if (wide) {
+                        st_global_v8(dst16 + c0, w);
+                        st_global_v8(dst16 + c0 + 16, w + 8);
+                    } else {
+#pragma unroll
+                        for (int t = 0; t < 16; t += 4)
+                            *reinterpret_cast<uint4*>(dst16 + c0 + 2 * t) = make_uint4(w[t], w[t + 1], w[t + 2], w[t + 3]);
+                    }
+                } else {
+#pragma unroll
+                    for (int t = 0; t < 32; t += 8) {
+                        uint32_t w[8];
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) w[e] = __float_as_uint(__uint_as_float(ov[h][t + e]) * inv);
+                        st_global_v8(dst + c0 + t, w);
+                    }
+                }
             }
         }
         tc_fence_before();
