@@ -121,6 +121,16 @@ def test_random_forests(seed, heads):
     run_and_compare(s, flags=FLAG_SETS[seed % 4])
 
 
+@pytest.mark.parametrize("heads", [workloads.Heads(32, 2, 64), workloads.Heads(24, 2, 128)])
+def test_gqa_groups_wider_than_eight(heads):
+    # g = 16 and 12 q heads per kv head: 128-row tensor units hold 8 and 10
+    # occurrences, 64-row mma.sync units 4 and 5
+    s = workloads.random_tree(seed=7, heads=heads, n_prompts=2, max_depth=4,
+                              prompt_range=(1, 300), seg_range=(1, 150))
+    for flags in FLAG_SETS:
+        run_and_compare(s, flags)
+
+
 @pytest.mark.parametrize("flags", FLAG_SETS)
 def test_qwen7b_shape_reduced(flags):
     # two prompts: ragged prompt lengths, 512-token segments, rows 112/56/28/14/7

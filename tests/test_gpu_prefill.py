@@ -34,7 +34,7 @@ def _src(script):
     return src
 
 
-def run_prefill(script, nodes_sid, counts, rows=None, seed=0, flags=0):
+def run_prefill(script, nodes_sid, counts, rows=None, seed=0, flags=0, o_offset=0):
     h = script.heads
     f = tp.Forest(h.num_q_heads, h.num_kv_heads, h.head_dim, pool_blocks=script.upper_bound_blocks(32) + 64,
                   device=DEV)
@@ -42,7 +42,10 @@ def run_prefill(script, nodes_sid, counts, rows=None, seed=0, flags=0):
     total = sum(counts)
     g = torch.Generator(device="cpu").manual_seed(seed)
     Q = torch.randn(total, h.num_q_heads, h.head_dim, generator=g).to(torch.bfloat16).to(DEV)
-    O = torch.empty_like(Q)
+    # o_offset elements into a larger buffer: an O that is 16-byte but not
+    # 32-byte aligned takes the kernel's 16-byte store path
+    O_buf = torch.empty(Q.numel() + o_offset, dtype=torch.bfloat16, device=DEV)
+    O = O_buf[o_offset:].view(Q.shape)
     LSE = torch.empty(total, h.num_q_heads, dtype=torch.float32, device=DEV)
     tp.tp_prefill(f.handle, [ids[x] for x in nodes_sid], counts, Q, O, LSE, flags)
     f.sync()
@@ -105,6 +108,19 @@ def test_prefill_long_path_several_chunks(flags):
     rng = np.random.default_rng(1)
     rows = sorted(set([0, 1, 699] + [int(x) for x in rng.integers(0, 700, 60)]))
     run_prefill(s, list(s.leaves), [700], rows=rows, flags=flags)
+
+
+@pytest.mark.parametrize("flags", FLAGS)
+def test_prefill_output_16_byte_aligned_only(flags):
+    # the wide-tree case again (its row blocks write O directly and through
+    # the merge), with O 16 bytes past a 32-byte boundary
+    s = workloads.segment_prefill(seed=2, n_prompts=4, prompt_len=1024, fanout=4, seg_len=512)
+    counts = [512] * len(s.leaves)
+    total = sum(counts)
+    rng = np.random.default_rng(3)
+    rows = sorted(set([0, 511, 512, total - 1] + [int(x) for x in rng.integers(0, total, 64)]))
+    O, _ = run_prefill(s, list(s.leaves), counts, rows=rows, o_offset=8, flags=flags)
+    assert O.data_ptr() % 32 == 16
 
 
 def test_prefill_last_token_matches_decode():
