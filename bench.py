@@ -532,18 +532,23 @@ def bench_prefill(args):
     dec_ms = kt["decode"]["ms"] / max(kt["decode"]["launches"], 1)
     peak, kind = peaks("bf16_tflops")
     achieved = flops / (dec_ms / 1e3) / 1e12
-    # end to end: pinned host Q in, O and LSE back, every step
+    # end to end through the host-buffer call: pinned host Q in, O and LSE
+    # back, every step; calls back to back (the library overlaps a call's
+    # copies with its neighbours' attention), then one tp_sync
     Qh, Oh = Q.cpu().pin_memory(), torch.empty(O.shape, dtype=O.dtype, pin_memory=True)
     Lh = torch.empty(L.shape, dtype=L.dtype, pin_memory=True)
-    Qd = torch.empty_like(Q)
+    tp.tp_prefill_host(forest.handle, nodes, counts, Qh, Oh, Lh, args.flags)
+    forest.sync()
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        Qd.copy_(Qh, non_blocking=True)
-        tp.tp_prefill(forest.handle, nodes, counts, Qd, O, L, args.flags)
-        Oh.copy_(O, non_blocking=True)
-        Lh.copy_(L, non_blocking=True)
-        stream.synchronize()
+        tp.tp_prefill_host(forest.handle, nodes, counts, Qh, Oh, Lh, args.flags)
+    forest.sync()
     e2e_s = (time.perf_counter() - t0) / args.steps
+    t0 = time.perf_counter()
+    for _ in range(args.steps):  # the same with a wait after every call
+        tp.tp_prefill_host(forest.handle, nodes, counts, Qh, Oh, Lh, args.flags)
+        forest.sync()
+    e2e_sync_s = (time.perf_counter() - t0) / args.steps
     line = {
         "metric": "tree prefill query tokens/s (causal multi-query attention over root-to-node paths); "
                   "TFLOP/s vs GB300 bf16 peak",
@@ -561,7 +566,9 @@ def bench_prefill(args):
                      "peak_source": f"{kind} bf16_tflops (burst)"},
         "kernel_ms_per_step": {"attention": dec_ms, "merge": kt["merge"]["ms"] / max(kt["merge"]["launches"], 1)},
         "e2e": {"value": total / e2e_s, "unit": "query-tokens/s", "h2d_bytes_per_step": Q.numel() * 2,
-                "d2h_bytes_per_step": O.numel() * 2 + L.numel() * 4},
+                "d2h_bytes_per_step": O.numel() * 2 + L.numel() * 4,
+                "call": "tp_prefill_host, calls back to back then tp_sync",
+                "value_wait_each_call": total / e2e_sync_s},
         "gpu_launches": int(kt["decode"]["launches"] + kt["merge"]["launches"]), "clocks": clocks,
     }
     if not args.no_cpu_baseline:
@@ -771,31 +778,31 @@ def main():
     ms_noshare = timed(args.steps, tp.TP_DECODE_NO_SHARE)
     steps(2, args.flags)
 
-    # ---- end to end through the public API: pinned host Q in, O/LSE out
+    # ---- end to end through the host-buffer call: pinned host Q in, O and
+    # LSE back, every step; calls back to back (the library overlaps a call's
+    # copies with its neighbours' attention), then one tp_sync
     Qh = Q.cpu().pin_memory()
     Oh = torch.empty(O.shape, dtype=O.dtype, pin_memory=True)
     Lh = torch.empty(LSE.shape, dtype=LSE.dtype, pin_memory=True)
-    Qd = torch.empty_like(Q)
-
-    def e2e_step():
-        Qd.copy_(Qh, non_blocking=True)
-        tp.tp_decode_ex(forest.handle, leaves, Qd, O, LSE, args.flags)
-        Oh.copy_(O, non_blocking=True)
-        Lh.copy_(LSE, non_blocking=True)
-        stream.synchronize()
-
     for _ in range(2):
-        e2e_step()
+        tp.tp_decode_host(forest.handle, leaves, Qh, Oh, Lh, args.flags)
+    forest.sync()
     if world > 1:
         dist.barrier()
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        e2e_step()
-    e2e_s = time.perf_counter() - t0
+        tp.tp_decode_host(forest.handle, leaves, Qh, Oh, Lh, args.flags)
     forest.sync()
+    e2e_s = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    for _ in range(args.steps):  # the same with a wait after every call
+        tp.tp_decode_host(forest.handle, leaves, Qh, Oh, Lh, args.flags)
+        forest.sync()
+    e2e_sync_s = time.perf_counter() - t0
 
     # ---- max over ranks
-    ms_total, ms_uncached, ms_noshare, e2e_s = max_over_ranks([ms_total, ms_uncached, ms_noshare, e2e_s], dev)
+    ms_total, ms_uncached, ms_noshare, e2e_s, e2e_sync_s = max_over_ranks(
+        [ms_total, ms_uncached, ms_noshare, e2e_s, e2e_sync_s], dev)
     leaves_all = n * world
 
     if rank == 0:
@@ -833,7 +840,9 @@ def main():
             "sharing_speedup": ms_noshare / ms_total,
             "e2e": {"value": leaves_all * args.steps / e2e_s, "unit": UNIT,
                     "h2d_bytes_per_step": Q.numel() * Q.element_size(),
-                    "d2h_bytes_per_step": O.numel() * O.element_size() + LSE.numel() * LSE.element_size()},
+                    "d2h_bytes_per_step": O.numel() * O.element_size() + LSE.numel() * LSE.element_size(),
+                    "call": "tp_decode_host, calls back to back then tp_sync",
+                    "value_wait_each_call": leaves_all * args.steps / e2e_sync_s},
             "gpu_launches": int(dec["launches"] + mer["launches"]),
             "clocks": clocks,
             "setup_s": t_setup,

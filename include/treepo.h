@@ -234,9 +234,33 @@ tp_status tp_append_tokens(tp_tree* tree, const tp_node* nodes, int32_t n, const
 tp_status tp_prefill(tp_tree* tree, const tp_node* nodes, const int32_t* n_queries, int32_t n, const void* Q,
                      void* O, float* LSE, uint32_t flags);
 
-/* Wait for the tree's stream; TP_ERR_DEVICE if a kernel gave up a bounded
- * wait since the last tp_sync (the flag is then cleared), TP_ERR_CUDA on a
- * CUDA error. */
+/* tp_decode_ex and tp_prefill with HOST buffers: the same operation (decode
+ * attention over root-to-leaf paths, Sec. 2.3 and 4.3; causal prefill over
+ * root-to-node paths), the same leaves / nodes / n_queries / flags and the
+ * same row layouts, but Q_host, O_host and LSE_host are host memory. The
+ * library uploads Q into device staging of its own, runs the attention there
+ * and downloads O and LSE. Library engineering with no counterpart in the
+ * paper.
+ *
+ * Asynchronous, like every attention call: the copies and the kernels are
+ * enqueued and the call returns. Q_host must stay unchanged, and O_host /
+ * LSE_host unread, until tp_sync returns (tp_sync also waits for these
+ * copies). Consecutive host-buffer calls use two staging slots in turn, with
+ * the uploads and downloads on copy streams of their own, so a call's copies
+ * overlap the neighbouring calls' attention. Page-locked (pinned) host
+ * memory makes the copies asynchronous; pageable memory is accepted, but
+ * the CUDA runtime then stages it and the call may block. The staging grows
+ * to the largest call seen (2 x (Q + O + LSE) bytes) and is freed with the
+ * tree. Errors: those of tp_decode_ex / tp_prefill, TP_ERR_INVALID_ARG for a
+ * NULL host pointer, TP_ERR_OOM / TP_ERR_CUDA (staging, copies). */
+tp_status tp_decode_host(tp_tree* tree, const tp_node* leaves, int32_t n, const void* Q_host, void* O_host,
+                         float* LSE_host, uint32_t flags);
+tp_status tp_prefill_host(tp_tree* tree, const tp_node* nodes, const int32_t* n_queries, int32_t n,
+                          const void* Q_host, void* O_host, float* LSE_host, uint32_t flags);
+
+/* Wait for the tree's stream (and the copy streams of the host-buffer
+ * calls); TP_ERR_DEVICE if a kernel gave up a bounded wait since the last
+ * tp_sync (the flag is then cleared), TP_ERR_CUDA on a CUDA error. */
 tp_status tp_sync(tp_tree* tree);
 
 /* Message for the last failed call on `tree` (or of tp_tree_create when

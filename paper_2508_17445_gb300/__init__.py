@@ -24,7 +24,7 @@ __all__ = [
     "tp_sync", "tp_last_error", "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop",
     "tp_debug_path", "tp_debug_gather",
     "tp_debug_schedule", "tp_decode_noalloc", "tp_append_tokens", "tp_synth_tokens", "tp_branch_assign",
-    "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "tp_prefill", "tp_debug_prefill_schedule", "TpRolloutParams", "TpRolloutStats",
+    "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "tp_prefill", "tp_debug_prefill_schedule", "tp_decode_host", "tp_prefill_host", "TpRolloutParams", "TpRolloutStats",
     "TpRolloutProbe", "rollout_params", "TP_BRANCH_EVEN", "TP_BRANCH_LOGP_HIGH", "TP_BRANCH_LOGP_LOW",
     "EVENT_NAMES", "TP_SEG_EOS", "TP_SEG_BOXED", "TP_SEG_FAILED", "TP_SEG_MAX_DEPTH", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE", "TP_DECODE_TCGEN05", "TP_DECODE_ALL_TCGEN05", "TP_MMA_SYNC",
     "EXPORTED_SYMBOLS",
@@ -56,7 +56,7 @@ EXPORTED_SYMBOLS = (
     "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop", "tp_debug_path",
     "tp_debug_gather", "tp_debug_schedule", "tp_decode_noalloc", "tp_append_tokens", "tp_synth_tokens",
     "tp_branch_assign", "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "tp_prefill",
-    "tp_debug_prefill_schedule",
+    "tp_debug_prefill_schedule", "tp_decode_host", "tp_prefill_host",
 )
 
 
@@ -153,6 +153,8 @@ def load_library() -> ctypes.CDLL:
         "tp_advantage_workspace_bytes": (I64, [I32, I32]),
         "tp_tree_advantage": (I32, [P, I32, P, P, I32, P, P, P, I64, P]),
         "tp_prefill": (I32, [P, P, P, I32, P, P, P, U32]),
+        "tp_decode_host": (I32, [P, P, I32, P, P, P, U32]),
+        "tp_prefill_host": (I32, [P, P, P, I32, P, P, P, U32]),
         "tp_debug_prefill_schedule": (I32, [P, P, P, I32, U32, P, I64, P]),
     }
     for name, (res, args) in sig.items():
@@ -290,6 +292,30 @@ def tp_prefill(h, nodes: Sequence[int], n_queries: Sequence[int], Q, O, LSE, fla
     _check(h, load_library().tp_prefill(h, arr.ctypes.data if len(arr) else None,
                                         m.ctypes.data if len(m) else None, len(arr), _ptr(Q), _ptr(O), _ptr(LSE),
                                         flags))
+
+
+def _host_ptr(t) -> int:
+    if t.is_cuda or not t.is_contiguous():
+        raise ValueError("host-buffer calls take contiguous CPU tensors (pinned for overlap)")
+    return t.data_ptr()
+
+
+def tp_decode_host(h, leaves: Sequence[int], Q, O, LSE, flags: int = 0) -> None:
+    """tp_decode_ex with host Q/O/LSE (contiguous CPU tensors, ideally pinned);
+    asynchronous: read O and LSE after tp_sync."""
+    arr = _node_array(leaves)
+    _check(h, load_library().tp_decode_host(h, arr.ctypes.data if len(arr) else None, len(arr), _host_ptr(Q),
+                                            _host_ptr(O), _host_ptr(LSE), flags))
+
+
+def tp_prefill_host(h, nodes: Sequence[int], n_queries: Sequence[int], Q, O, LSE, flags: int = 0) -> None:
+    """tp_prefill with host Q/O/LSE (contiguous CPU tensors, ideally pinned);
+    asynchronous: read O and LSE after tp_sync."""
+    arr = _node_array(nodes)
+    m = np.ascontiguousarray(np.asarray(n_queries, dtype=np.int32).reshape(-1))
+    _check(h, load_library().tp_prefill_host(h, arr.ctypes.data if len(arr) else None,
+                                             m.ctypes.data if len(m) else None, len(arr), _host_ptr(Q),
+                                             _host_ptr(O), _host_ptr(LSE), flags))
 
 
 def _parse_schedule(w: np.ndarray) -> Dict[str, np.ndarray]:

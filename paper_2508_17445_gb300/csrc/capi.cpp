@@ -195,6 +195,17 @@ tp_status tp_tree_destroy(tp_tree* t) {
         if (t->h_pinned[k]) cudaFreeHost(t->h_pinned[k]);
         if (t->h_pinned_ev[k]) cudaEventDestroy(t->h_pinned_ev[k]);
     }
+    for (cudaStream_t s : {t->hp_h2d, t->hp_d2h})
+        if (s) {
+            cudaStreamSynchronize(s);
+            cudaStreamDestroy(s);
+        }
+    for (int k = 0; k < 2; ++k) {
+        for (cudaEvent_t e : {t->hp_up[k], t->hp_done[k], t->hp_down[k]})
+            if (e) cudaEventDestroy(e);
+        for (void* p : {t->hp_q[k], t->hp_o[k], t->hp_lse[k]})
+            if (p) cudaFree(p);
+    }
     delete t;
     return TP_OK;
 }
@@ -516,6 +527,92 @@ tp_status tp_prefill(tp_tree* t, const tp_node* nodes, const int32_t* n_queries,
     return run_schedule(t, S, Q, O, LSE);
 }
 
+}  // extern "C"
+
+namespace {
+// One host-buffer call: upload Q into staging slot b once the attention that
+// last read that slot has finished, run the attention there once the upload
+// has landed and the slot's previous results have been downloaded, then
+// download O and LSE. Consecutive calls alternate slots, so a call's upload
+// and download overlap the neighbouring calls' attention.
+template <typename Run>
+tp_status run_host(tp_tree* t, int64_t q_bytes, int64_t o_bytes, int64_t lse_bytes, const void* Qh, void* Oh,
+                   float* Lh, Run run) {
+    cudaError_t e = cudaSuccess;
+    if (!t->hp_h2d) {
+        e = cudaStreamCreateWithFlags(&t->hp_h2d, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&t->hp_d2h, cudaStreamNonBlocking);
+        for (int k = 0; k < 2 && e == cudaSuccess; ++k)
+            for (cudaEvent_t* ev : {&t->hp_up[k], &t->hp_done[k], &t->hp_down[k]})
+                if (e == cudaSuccess) e = cudaEventCreateWithFlags(ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) return cuda_fail(t, e, "host-buffer streams");
+    }
+    const int b = (int)(t->hp_calls & 1);
+    if (q_bytes > t->hp_q_cap[b] || o_bytes > t->hp_o_cap[b] || lse_bytes > t->hp_lse_cap[b]) {
+        // a slot grows: no copy of the other calls may still use it
+        e = cudaStreamSynchronize(t->hp_h2d);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(t->hp_d2h);
+        if (e != cudaSuccess) return cuda_fail(t, e, "host-buffer streams");
+    }
+    tp_status st = tp::ensure_device_bytes(t, &t->hp_q[b], &t->hp_q_cap[b], q_bytes, "query staging");
+    if (st == TP_OK) st = tp::ensure_device_bytes(t, &t->hp_o[b], &t->hp_o_cap[b], o_bytes, "output staging");
+    if (st == TP_OK) st = tp::ensure_device_bytes(t, &t->hp_lse[b], &t->hp_lse_cap[b], lse_bytes, "LSE staging");
+    if (st != TP_OK) return st;
+    e = cudaStreamWaitEvent(t->hp_h2d, t->hp_done[b], 0);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(t->hp_q[b], Qh, (size_t)q_bytes, cudaMemcpyHostToDevice, t->hp_h2d);
+    if (e == cudaSuccess) e = cudaEventRecord(t->hp_up[b], t->hp_h2d);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(t->stream, t->hp_up[b], 0);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(t->stream, t->hp_down[b], 0);
+    if (e != cudaSuccess) return cuda_fail(t, e, "query upload");
+    st = run(t->hp_q[b], t->hp_o[b], (float*)t->hp_lse[b]);
+    if (st != TP_OK) return st;
+    e = cudaEventRecord(t->hp_done[b], t->stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(t->hp_d2h, t->hp_done[b], 0);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(Oh, t->hp_o[b], (size_t)o_bytes, cudaMemcpyDeviceToHost, t->hp_d2h);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(Lh, t->hp_lse[b], (size_t)lse_bytes, cudaMemcpyDeviceToHost, t->hp_d2h);
+    if (e == cudaSuccess) e = cudaEventRecord(t->hp_down[b], t->hp_d2h);
+    if (e != cudaSuccess) return cuda_fail(t, e, "result download");
+    ++t->hp_calls;
+    return TP_OK;
+}
+}  // namespace
+
+extern "C" {
+
+tp_status tp_decode_host(tp_tree* t, const tp_node* leaves, int32_t n, const void* Q_host, void* O_host,
+                         float* LSE_host, uint32_t flags) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    if (n < 0) return fail(t, TP_ERR_INVALID_ARG, "n < 0");
+    if (n == 0) return TP_OK;
+    if (!leaves) return fail(t, TP_ERR_INVALID_ARG, "leaves is NULL");
+    if (!t->cfg.pool) return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree cannot decode");
+    if (!Q_host || !O_host || !LSE_host) return fail(t, TP_ERR_INVALID_ARG, "Q/O/LSE host pointer is NULL");
+    const int64_t row = (int64_t)t->cfg.num_q_heads * t->cfg.head_dim;
+    return run_host(t, n * row * 2, n * row * 2, (int64_t)n * t->cfg.num_q_heads * 4, Q_host, O_host, LSE_host,
+                    [&](const void* Q, void* O, float* LSE) { return tp_decode_ex(t, leaves, n, Q, O, LSE, flags); });
+}
+
+tp_status tp_prefill_host(tp_tree* t, const tp_node* nodes, const int32_t* n_queries, int32_t n, const void* Q_host,
+                          void* O_host, float* LSE_host, uint32_t flags) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    if (n < 0) return fail(t, TP_ERR_INVALID_ARG, "n < 0");
+    if (n == 0) return TP_OK;
+    if (!nodes || !n_queries) return fail(t, TP_ERR_INVALID_ARG, "nodes or n_queries is NULL");
+    if (!t->cfg.pool) return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree cannot run attention");
+    if (!Q_host || !O_host || !LSE_host) return fail(t, TP_ERR_INVALID_ARG, "Q/O/LSE host pointer is NULL");
+    int64_t total = 0;
+    for (int32_t i = 0; i < n; ++i) {
+        if (n_queries[i] < 0) return fail(t, TP_ERR_INVALID_ARG, "n_queries[i] < 0");
+        total += n_queries[i];
+    }
+    if (total == 0) return TP_OK;
+    const int64_t row = (int64_t)t->cfg.num_q_heads * t->cfg.head_dim;
+    return run_host(t, total * row * 2, total * row * 2, total * t->cfg.num_q_heads * 4, Q_host, O_host, LSE_host,
+                    [&](const void* Q, void* O, float* LSE) {
+                        return tp_prefill(t, nodes, n_queries, n, Q, O, LSE, flags);
+                    });
+}
+
 tp_status tp_debug_prefill_schedule(tp_tree* t, const tp_node* nodes, const int32_t* n_queries, int32_t n,
                                     uint32_t flags, int32_t* buf, int64_t cap, int64_t* len) {
     if (!t || !len) return TP_ERR_INVALID_ARG;
@@ -708,6 +805,8 @@ tp_status tp_sync(tp_tree* t) {
     if (!t) return TP_ERR_INVALID_ARG;
     if (!t->cfg.pool) return TP_OK;
     cudaError_t e = cudaStreamSynchronize(t->stream);
+    if (e == cudaSuccess && t->hp_h2d) e = cudaStreamSynchronize(t->hp_h2d);
+    if (e == cudaSuccess && t->hp_d2h) e = cudaStreamSynchronize(t->hp_d2h);
     if (e != cudaSuccess) return cuda_fail(t, e, "cudaStreamSynchronize");
     int32_t flag = 0;
     e = cudaMemcpy(&flag, t->d_err, sizeof flag, cudaMemcpyDeviceToHost);

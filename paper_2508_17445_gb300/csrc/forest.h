@@ -262,6 +262,19 @@ struct tp_tree {
     cudaStream_t side = nullptr;  // second stream for concurrent tcgen05 units
     cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
 
+    // host-buffer calls (tp_decode_host, tp_prefill_host): two staging slots
+    // used in turn, uploads and downloads on streams of their own so that a
+    // call's copies overlap its neighbours' attention
+    cudaStream_t hp_h2d = nullptr, hp_d2h = nullptr;
+    cudaEvent_t hp_up[2] = {nullptr, nullptr};    // slot's Q uploaded
+    cudaEvent_t hp_done[2] = {nullptr, nullptr};  // slot's attention finished
+    cudaEvent_t hp_down[2] = {nullptr, nullptr};  // slot's O and LSE downloaded
+    void* hp_q[2] = {nullptr, nullptr};
+    void* hp_o[2] = {nullptr, nullptr};
+    void* hp_lse[2] = {nullptr, nullptr};
+    int64_t hp_q_cap[2] = {0, 0}, hp_o_cap[2] = {0, 0}, hp_lse_cap[2] = {0, 0};  // bytes
+    uint64_t hp_calls = 0;
+
     // kernel timing (tp_profile_start / tp_profile_stop)
     bool profiling = false;
     std::vector<cudaEvent_t> ev_pool;

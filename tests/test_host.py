@@ -231,6 +231,26 @@ class _FakePtr:
         return 0x1000
 
 
+def test_host_buffer_calls_check_their_arguments():
+    import torch
+    f = meta_forest(pool_blocks=8)
+    r = f.add_root()
+    tp.tp_append_segment(f.handle, r, 40)
+    q = torch.zeros(1, f.cfg.num_q_heads, f.cfg.head_dim, dtype=torch.bfloat16)
+    o, lse = torch.empty_like(q), torch.empty(1, f.cfg.num_q_heads)
+    for call in (lambda: tp.tp_decode_host(f.handle, [r], q, o, lse),
+                 lambda: tp.tp_prefill_host(f.handle, [r], [1], q, o, lse)):
+        with pytest.raises(tp.TreepoError) as e:   # metadata-only trees run no attention
+            call()
+        assert e.value.code == "INVALID_ARG"
+    lib = tp.load_library()
+    nodes = np.array([r], dtype=np.int32)
+    assert lib.tp_decode_host(f.handle, nodes.ctypes.data, 0, None, None, None, 0) == 0   # n = 0: nothing to do
+    assert lib.tp_decode_host(f.handle, nodes.ctypes.data, -1, None, None, None, 0) == -1
+    with pytest.raises(ValueError):   # the binding takes contiguous CPU tensors only
+        tp.tp_decode_host(f.handle, [r], q.transpose(1, 2), o, lse)
+
+
 def test_fork_of_frozen_node_adds_children():
     f = meta_forest()
     r = f.add_root()
