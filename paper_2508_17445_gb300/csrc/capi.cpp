@@ -61,6 +61,122 @@ tp_status stage_upload(tp_tree* t, int32_t* dst, const int32_t* src, int64_t wor
     return TP_OK;
 }
 
+// Host half of appending one token to each of nodes[0..n): the checks, a new
+// block for every node whose last block is full (*need of them), and the pool
+// slot of each new token in t->tok_slots. Nothing changes on failure.
+tp_status append_tokens_plan(tp_tree* t, const tp_node* nodes, int32_t n, int64_t* need_out) {
+    SchedScratch& X = t->scratch;
+    if (X.mark.size() < t->nodes.size()) {
+        X.mark.resize(t->nodes.size(), 0);
+        X.local.resize(t->nodes.size(), 0);
+    }
+    if (++X.epoch == 0) {
+        std::fill(X.mark.begin(), X.mark.end(), 0u);
+        X.epoch = 1;
+    }
+    const int32_t bt = t->cfg.block_tokens;
+    int64_t need = 0;
+    for (int32_t i = 0; i < n; ++i) {
+        tp_status st = check_live(t, nodes[i], false);
+        if (st != TP_OK) return st;
+        const Node& nd = t->nodes[(size_t)nodes[i]];
+        if (nd.state != 0) return fail(t, TP_ERR_FROZEN, "node " + std::to_string(nodes[i]) + " has been forked");
+        if (X.mark[(size_t)nodes[i]] == X.epoch)
+            return fail(t, TP_ERR_INVALID_ARG, "node " + std::to_string(nodes[i]) + " is listed twice");
+        if (nd.n_tokens >= INT32_MAX / 2) return fail(t, TP_ERR_INVALID_ARG, "node too long");
+        X.mark[(size_t)nodes[i]] = X.epoch;
+        need += nd.n_tokens % bt == 0;
+    }
+    if (need > t->pool.free_count())
+        return fail(t, TP_ERR_OOM, "pool exhausted: need " + std::to_string(need) + " blocks, " +
+                                       std::to_string(t->pool.free_count()) + " free");
+    std::vector<int32_t>& slots = t->tok_slots;
+    slots.resize((size_t)n);
+    for (int32_t i = 0; i < n; ++i) {
+        Node& nd = t->nodes[(size_t)nodes[i]];
+        if (nd.n_tokens % bt == 0) t->pool.alloc(1, nd.blocks);  // cannot fail: counted above
+        slots[(size_t)i] = nd.blocks[(size_t)(nd.n_tokens / bt)] * bt + nd.n_tokens % bt;
+    }
+    *need_out = need;
+    return TP_OK;
+}
+
+// Undoes append_tokens_plan's block allocations (before the commit).
+void append_tokens_unplan(tp_tree* t, const tp_node* nodes, int32_t n) {
+    const int32_t bt = t->cfg.block_tokens;
+    for (int32_t i = 0; i < n; ++i) {
+        Node& nd = t->nodes[(size_t)nodes[i]];
+        if (nd.n_tokens % bt == 0) {
+            t->pool.release({nd.blocks.back()});
+            nd.blocks.pop_back();
+        }
+    }
+}
+
+void append_tokens_commit(tp_tree* t, const tp_node* nodes, int32_t n, int64_t need) {
+    for (int32_t i = 0; i < n; ++i) ++t->nodes[(size_t)nodes[i]].n_tokens;
+    ++t->version;
+    if (need > 0) ++t->struct_version;
+}
+
+// One token step of the rollout's decode loop in one upload and one launch:
+// append a token to each of nodes[0..n) with the stand-in activations of
+// (seed, pos), Q of the rows into q; and, when the cached decode schedule is
+// the one for exactly these nodes and the append stays inside their last
+// blocks, the schedule patch the next tp_decode_ex(decode_flags) would apply.
+// d_buf: device int32 scratch of at least 4 n words.
+tp_status rollout_token_step(tp_tree* t, const tp_node* nodes, int32_t n, int32_t* d_buf, int64_t buf_words,
+                             uint64_t seed, int32_t pos, uint16_t* q, uint32_t decode_flags) {
+    if (n == 0) return TP_OK;
+    int64_t need = 0;
+    tp_status st = append_tokens_plan(t, nodes, n, &need);
+    if (st != TP_OK) return st;
+    const uint32_t key = decode_flags & ~TP_DECODE_NO_CACHE;
+    const bool patch = !(decode_flags & TP_DECODE_NO_CACHE) && need == 0 && t->sched_valid &&
+                       t->sched_flags == key && t->sched_version == t->version &&
+                       t->sched_struct == t->struct_version && t->sched_leaves.size() == (size_t)n &&
+                       std::equal(nodes, nodes + n, t->sched_leaves.begin()) &&
+                       2 * (int64_t)n + (int64_t)t->sched.leaf_tail.size() <= buf_words;
+    append_tokens_commit(t, nodes, n, need);
+    const int32_t n_pairs = patch ? patch_schedule(t, t->sched, t->patch_words) : 0;
+    std::vector<int32_t>& w = t->scratch.step_words;  // row nodes | pool slots | patch pairs
+    w.assign(nodes, nodes + n);
+    w.insert(w.end(), t->tok_slots.begin(), t->tok_slots.end());
+    if (n_pairs > 0) w.insert(w.end(), t->patch_words.begin(), t->patch_words.begin() + 2 * (int64_t)n_pairs);
+    st = (int64_t)w.size() <= buf_words ? stage_upload(t, d_buf, w.data(), (int64_t)w.size())
+                                        : fail(t, TP_ERR_INVALID_ARG, "rollout step buffer too small");
+    if (st == TP_OK) {
+        StepArgs a;
+        a.row_node = d_buf;
+        a.slots = d_buf + n;
+        a.pairs = d_buf + 2 * n;
+        a.sched = t->d_sched;
+        a.pool = (uint8_t*)t->cfg.pool;
+        a.q = q;
+        a.seed = seed;
+        a.head_bytes = t->cfg.block_tokens * t->cfg.head_dim * 2;
+        a.block_bytes = (int64_t)2 * t->cfg.num_kv_heads * a.head_bytes;
+        a.hkv = t->cfg.num_kv_heads;
+        a.q_width = t->cfg.num_q_heads * t->cfg.head_dim;
+        a.pos = pos;
+        a.n = n;
+        a.n_pairs = n_pairs;
+        LaunchTimer timer(t, KK_APPEND);
+        cudaError_t e = launch_rollout_step(t->cfg.head_dim, a, t->stream);
+        if (e != cudaSuccess) st = cuda_fail(t, e, "rollout step kernel");
+    }
+    if (st != TP_OK) {  // back to the state before the call; the cached schedule is rebuilt next time
+        for (int32_t i = 0; i < n; ++i) --t->nodes[(size_t)nodes[i]].n_tokens;
+        append_tokens_unplan(t, nodes, n);
+        --t->version;
+        if (need > 0) --t->struct_version;
+        t->sched_valid = false;
+        return st;
+    }
+    if (patch) t->sched_version = t->version;
+    return TP_OK;
+}
+
 }  // namespace tp
 
 namespace {
@@ -298,42 +414,13 @@ tp_status tp_append_tokens(tp_tree* t, const tp_node* nodes, int32_t n, const vo
     } else if (K || V) {
         return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree: K and V must be NULL");
     }
-    tp::SchedScratch& X = t->scratch;
-    if (X.mark.size() < t->nodes.size()) {
-        X.mark.resize(t->nodes.size(), 0);
-        X.local.resize(t->nodes.size(), 0);
-    }
-    if (++X.epoch == 0) {
-        std::fill(X.mark.begin(), X.mark.end(), 0u);
-        X.epoch = 1;
-    }
-    const int32_t bt = t->cfg.block_tokens;
     int64_t need = 0;
-    for (int32_t i = 0; i < n; ++i) {
-        tp_status st = tp::check_live(t, nodes[i], false);
-        if (st != TP_OK) return st;
-        const tp::Node& nd = t->nodes[(size_t)nodes[i]];
-        if (nd.state != 0) return fail(t, TP_ERR_FROZEN, "node " + std::to_string(nodes[i]) + " has been forked");
-        if (X.mark[(size_t)nodes[i]] == X.epoch)
-            return fail(t, TP_ERR_INVALID_ARG, "node " + std::to_string(nodes[i]) + " is listed twice");
-        if (nd.n_tokens >= INT32_MAX / 2) return fail(t, TP_ERR_INVALID_ARG, "node too long");
-        X.mark[(size_t)nodes[i]] = X.epoch;
-        need += nd.n_tokens % bt == 0;
-    }
-    if (need > t->pool.free_count())
-        return fail(t, TP_ERR_OOM, "pool exhausted: need " + std::to_string(need) + " blocks, " +
-                                       std::to_string(t->pool.free_count()) + " free");
-    std::vector<int32_t>& slots = t->tok_slots;
-    slots.resize((size_t)n);
-    for (int32_t i = 0; i < n; ++i) {
-        tp::Node& nd = t->nodes[(size_t)nodes[i]];
-        if (nd.n_tokens % bt == 0) t->pool.alloc(1, nd.blocks);  // cannot fail: counted above
-        slots[(size_t)i] = nd.blocks[(size_t)(nd.n_tokens / bt)] * bt + nd.n_tokens % bt;
-    }
+    tp_status st = tp::append_tokens_plan(t, nodes, n, &need);
+    if (st != TP_OK) return st;
     if (t->cfg.pool) {
-        tp_status st = ensure_device(t, t->d_tok_slots, t->d_tok_slots_cap, n, "token slot buffer");
-        if (st == TP_OK) st = stage_upload(t, t->d_tok_slots, slots.data(), n);
-        cudaError_t e = cudaSuccess;
+        const int32_t bt = t->cfg.block_tokens;
+        st = ensure_device(t, t->d_tok_slots, t->d_tok_slots_cap, n, "token slot buffer");
+        if (st == TP_OK) st = stage_upload(t, t->d_tok_slots, t->tok_slots.data(), n);
         if (st == TP_OK) {
             tp::AppendTokensArgs a;
             a.k = K;
@@ -345,23 +432,15 @@ tp_status tp_append_tokens(tp_tree* t, const tp_node* nodes, int32_t n, const vo
             a.hkv = t->cfg.num_kv_heads;
             a.n = n;
             tp::LaunchTimer timer(t, tp::KK_APPEND);
-            e = tp::launch_append_tokens(t->cfg.head_dim, a, t->stream);
+            cudaError_t e = tp::launch_append_tokens(t->cfg.head_dim, a, t->stream);
             if (e != cudaSuccess) st = cuda_fail(t, e, "token append kernel");
         }
-        if (st != TP_OK) {  // undo the block allocations
-            for (int32_t i = 0; i < n; ++i) {
-                tp::Node& nd = t->nodes[(size_t)nodes[i]];
-                if (nd.n_tokens % bt == 0) {
-                    t->pool.release({nd.blocks.back()});
-                    nd.blocks.pop_back();
-                }
-            }
+        if (st != TP_OK) {
+            tp::append_tokens_unplan(t, nodes, n);
             return st;
         }
     }
-    for (int32_t i = 0; i < n; ++i) ++t->nodes[(size_t)nodes[i]].n_tokens;
-    ++t->version;
-    if (need > 0) ++t->struct_version;
+    tp::append_tokens_commit(t, nodes, n, need);
     return TP_OK;
 }
 

@@ -138,6 +138,21 @@ struct SynthArgs {
     int32_t pos0;
 };
 
+// One token step of the rollout's decode loop (rollout_token_step): the
+// stand-in activations of each row's new token, K and V written straight
+// into the row's pool slot, Q into q; then the decode schedule's patches.
+struct StepArgs {
+    const int32_t* row_node;  // [n] node of each row
+    const int32_t* slots;     // [n] pool slot of each row's new token
+    const int32_t* pairs;     // [2 n_pairs]: (schedule word index, new value)
+    int32_t* sched;
+    uint8_t* pool;
+    uint16_t* q;              // [n][q_width]
+    uint64_t seed;
+    int64_t block_bytes;
+    int32_t head_bytes, hkv, q_width, pos, n, n_pairs;
+};
+
 // Tree advantage (Eq. tree_ae) over a node table; see tp_tree_advantage.
 struct AdvantageArgs {
     const int32_t* parent;  // [n_nodes]
@@ -164,6 +179,7 @@ cudaError_t launch_gather(int head_dim, const GatherArgs& a, int64_t n_tokens, c
 cudaError_t launch_patch(int32_t* sched, const int32_t* pairs, int32_t n, cudaStream_t s);
 cudaError_t launch_append_tokens(int head_dim, const AppendTokensArgs& a, cudaStream_t s);
 cudaError_t launch_synth(const SynthArgs& a, cudaStream_t s);
+cudaError_t launch_rollout_step(int head_dim, const StepArgs& a, cudaStream_t s);
 cudaError_t launch_advantage(const AdvantageArgs& a, cudaStream_t s);
 int decode_smem_bytes(int head_dim);
 // Device address of the library's static scratch array (tp_decode_noalloc).
@@ -229,6 +245,7 @@ struct SchedScratch {
     std::vector<int32_t> units[3], sorted, bucket;
     std::vector<int32_t> pair_occ, pair_slot, merge_off, merge_pos, merge_slot;
     std::vector<int32_t> tile_pos, node_tile_off, vis;  // prefill
+    std::vector<int32_t> step_words;                    // rollout_token_step's upload
 };
 
 }  // namespace tp
@@ -325,6 +342,11 @@ tp_status ensure_device_bytes(tp_tree* t, void** ptr, int64_t* cap, int64_t need
 // double-buffered pinned staging area; a staging buffer is reused only after
 // its previous copy has completed.
 tp_status stage_upload(tp_tree* t, int32_t* dst, const int32_t* src, int64_t words);
+tp_status append_tokens_plan(tp_tree* t, const tp_node* nodes, int32_t n, int64_t* need);
+void append_tokens_unplan(tp_tree* t, const tp_node* nodes, int32_t n);
+void append_tokens_commit(tp_tree* t, const tp_node* nodes, int32_t n, int64_t need);
+tp_status rollout_token_step(tp_tree* t, const tp_node* nodes, int32_t n, int32_t* d_buf, int64_t buf_words,
+                             uint64_t seed, int32_t pos, uint16_t* q, uint32_t decode_flags);
 
 // forest.cpp
 tp_status fail(tp_tree* t, tp_status code, const std::string& msg);

@@ -241,6 +241,14 @@ __global__ void append_tokens_kernel(const AppendTokensArgs a) {
 }
 
 // ------------------------------------------------------ stand-in activations --
+// A 64-bit draw -> 4 consecutive bf16 values (low 16 bits first), as two
+// 32-bit words of bf16 pairs.
+__device__ __forceinline__ uint2 synth_words(uint64_t h) {
+    const uint32_t lo = synth_bf16_bits((uint32_t)h & 0xffffu) | (uint32_t)synth_bf16_bits((uint32_t)(h >> 16) & 0xffffu) << 16;
+    const uint32_t hi = synth_bf16_bits((uint32_t)(h >> 32) & 0xffffu) | (uint32_t)synth_bf16_bits((uint32_t)(h >> 48)) << 16;
+    return make_uint2(lo, hi);
+}
+
 // One thread per 64-bit draw = 4 consecutive bf16 values of one row.
 __global__ void synth_kernel(const SynthArgs a) {
     const int kv_words = a.kv_width / 4, q_words = a.q_width / 4;
@@ -267,9 +275,48 @@ __global__ void synth_kernel(const SynthArgs a) {
         const uint32_t node = (uint32_t)(a.row_node ? a.row_node[i] : a.node0);
         const uint32_t pos = (uint32_t)(a.row_node ? a.pos0 : a.pos0 + i);
         const uint64_t h = splitmix64(a.seed, draw_counter(tag, node, pos, (uint32_t)w));
-        const uint32_t lo = synth_bf16_bits((uint32_t)h & 0xffffu) | (uint32_t)synth_bf16_bits((uint32_t)(h >> 16) & 0xffffu) << 16;
-        const uint32_t hi = synth_bf16_bits((uint32_t)(h >> 32) & 0xffffu) | (uint32_t)synth_bf16_bits((uint32_t)(h >> 48)) << 16;
-        *reinterpret_cast<uint2*>(out + i * width + 4 * w) = make_uint2(lo, hi);
+        *reinterpret_cast<uint2*>(out + i * width + 4 * w) = synth_words(h);
+    }
+}
+
+// One token step of the rollout's decode loop: row i's new token (node
+// row_node[i], position pos) gets the stand-in activations synth_kernel
+// would draw for it, K and V written straight into its pool slot (the bytes
+// append_tokens_kernel would write), Q into q; then the schedule words the
+// append changed are patched. One thread per 16-byte K/V chunk (two draws),
+// per Q draw, per patch.
+template <int HD>
+__global__ void rollout_step_kernel(const StepArgs a) {
+    constexpr int CH = HD / 8;
+    const int64_t kv_items = (int64_t)a.n * 2 * a.hkv * CH;
+    const int q_words = a.q_width / 4;
+    const int64_t q_items = (int64_t)a.n * q_words;
+    const int64_t total = kv_items + q_items + a.n_pairs;
+    for (int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; idx < total;
+         idx += (int64_t)gridDim.x * blockDim.x) {
+        if (idx < kv_items) {
+            const int c = (int)(idx % CH);
+            const int h = (int)((idx / CH) % a.hkv);
+            const int kv = (int)((idx / ((int64_t)CH * a.hkv)) & 1);
+            const int i = (int)(idx / ((int64_t)CH * a.hkv * 2));
+            const uint32_t node = (uint32_t)a.row_node[i], tag = kv ? kTagV : kTagK;
+            const uint32_t w0 = (uint32_t)(h * (HD / 4) + 2 * c);  // the chunk's two draws of the row
+            const uint2 x0 = synth_words(splitmix64(a.seed, draw_counter(tag, node, (uint32_t)a.pos, w0)));
+            const uint2 x1 = synth_words(splitmix64(a.seed, draw_counter(tag, node, (uint32_t)a.pos, w0 + 1)));
+            const int32_t slot = a.slots[i];
+            uint8_t* dst = a.pool + (int64_t)(slot / kBlockTokens) * a.block_bytes +
+                           (int64_t)(kv * a.hkv + h) * a.head_bytes + kv_off<kBlockTokens>(slot % kBlockTokens, c);
+            *reinterpret_cast<uint4*>(dst) = make_uint4(x0.x, x0.y, x1.x, x1.y);
+        } else if (idx < kv_items + q_items) {
+            const int64_t r = idx - kv_items;
+            const int i = (int)(r / q_words), w = (int)(r % q_words);
+            const uint32_t node = (uint32_t)a.row_node[i];
+            *reinterpret_cast<uint2*>(a.q + (int64_t)i * a.q_width + 4 * w) =
+                synth_words(splitmix64(a.seed, draw_counter(kTagQ, node, (uint32_t)a.pos, (uint32_t)w)));
+        } else {
+            const int64_t k = idx - kv_items - q_items;
+            a.sched[a.pairs[2 * k]] = a.pairs[2 * k + 1];
+        }
     }
 }
 
@@ -2062,6 +2109,17 @@ cudaError_t launch_append_tokens(int hd, const AppendTokensArgs& a, cudaStream_t
         append_tokens_kernel<64><<<grid, 256, 0, s>>>(a);
     else
         append_tokens_kernel<128><<<grid, 256, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_rollout_step(int hd, const StepArgs& a, cudaStream_t s) {
+    const int64_t items = (int64_t)a.n * (2 * a.hkv * (hd / 8) + a.q_width / 4) + a.n_pairs;
+    if (items == 0) return cudaSuccess;
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((items + 255) / 256, 152 * 16));
+    if (hd == 64)
+        rollout_step_kernel<64><<<grid, 256, 0, s>>>(a);
+    else
+        rollout_step_kernel<128><<<grid, 256, 0, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -128,7 +128,7 @@ class Rollout {
     std::vector<Path> queue_;
     std::vector<Segment> seg_;
     DevBuf k_, v_, q_, o_, lse_, rows_;
-    std::vector<int32_t> gen_, gen_prev_, counts_;
+    std::vector<int32_t> gen_, counts_;
     std::vector<double> frac_, logp_;
     std::vector<int32_t> order_, split_;
 
@@ -207,33 +207,18 @@ Segment Rollout::draw_segment(int32_t node) const {
 // Token-synchronous generation: token t of every path whose segment is longer
 // than t is appended, then those paths decode.
 tp_status Rollout::decode_tokens() {
-    const int32_t kvw = t_->cfg.num_kv_heads * t_->cfg.head_dim, qw = t_->cfg.num_q_heads * t_->cfg.head_dim;
+    const int32_t qw = t_->cfg.num_q_heads * t_->cfg.head_dim;
     int32_t max_len = 0;
     for (const Segment& s : seg_) max_len = std::max(max_len, s.len);
-    gen_prev_.clear();
     for (int32_t t = 0; t < max_len; ++t) {
         gen_.clear();
         for (size_t i = 0; i < queue_.size(); ++i)
             if (seg_[i].len > t) gen_.push_back(queue_[i].node);
         const int32_t n = (int32_t)gen_.size();
-        if (gen_ != gen_prev_) {
-            tp_status s = tp::stage_upload(t_, (int32_t*)rows_.p, gen_.data(), n);
-            if (s != TP_OK) return s;
-            gen_prev_ = gen_;
-        }
-        tp::SynthArgs a{};
-        a.k = (uint16_t*)k_.p;
-        a.v = (uint16_t*)v_.p;
-        a.q = (uint16_t*)q_.p;
-        a.row_node = (const int32_t*)rows_.p;
-        a.seed = p_.seed;
-        a.rows = n;
-        a.kv_width = kvw;
-        a.q_width = qw;
-        a.pos0 = t;
-        cudaError_t e = tp::launch_synth(a, t_->stream);
-        if (e != cudaSuccess) return tp::cuda_fail(t_, e, "synth kernel");
-        tp_status s = tp_append_tokens(t_, gen_.data(), n, k_.p, v_.p);
+        // the token's stand-in activations straight into the pool, Q into q_,
+        // and the cached decode schedule patched: one upload, one launch
+        tp_status s = tp::rollout_token_step(t_, gen_.data(), n, (int32_t*)rows_.p, rows_.cap / 4, p_.seed, t,
+                                             (uint16_t*)q_.p, p_.decode_flags);
         if (s != TP_OK) return s;
         note_pool();
         s = tp_decode_ex(t_, gen_.data(), n, q_.p, o_.p, (float*)lse_.p, p_.decode_flags);
@@ -241,7 +226,7 @@ tp_status Rollout::decode_tokens() {
         if (probe_ && probe_->call == st_.decode_calls) {
             const int32_t rows = std::min(n, probe_->cap);
             if (probe_->o) {
-                e = cudaMemcpyAsync(probe_->o, o_.p, (size_t)rows * qw * 2, cudaMemcpyDeviceToDevice, t_->stream);
+                cudaError_t e = cudaMemcpyAsync(probe_->o, o_.p, (size_t)rows * qw * 2, cudaMemcpyDeviceToDevice, t_->stream);
                 if (e == cudaSuccess && probe_->lse)
                     e = cudaMemcpyAsync(probe_->lse, lse_.p, (size_t)rows * t_->cfg.num_q_heads * 4,
                                         cudaMemcpyDeviceToDevice, t_->stream);
@@ -295,7 +280,7 @@ tp_status Rollout::run(tp_rollout_stats* stats) {
         if (s == TP_OK && p.decode) s = grow(q_, rows_max * qw * 2, "rollout Q");
         if (s == TP_OK && p.decode) s = grow(o_, rows_max * qw * 2, "rollout O");
         if (s == TP_OK && p.decode) s = grow(lse_, rows_max * t_->cfg.num_q_heads * 4, "rollout LSE");
-        if (s == TP_OK && p.decode) s = grow(rows_, rows_max * 4, "rollout row nodes");
+        if (s == TP_OK && p.decode) s = grow(rows_, rows_max * 16, "rollout token-step words");
         if (s != TP_OK) return s;
     }
     qs_.assign((size_t)nq, QueryState());
