@@ -287,11 +287,15 @@ typedef struct {
 tp_status tp_get_stats(tp_tree* tree, tp_stats* out);
 
 /* ---- kernel timing ------------------------------------------------------
- * While profiling is on, every kernel the library launches is bracketed by a
- * pair of CUDA events recorded on the tree's stream. tp_profile_stop waits
- * for the stream and returns, per kernel kind, the launch count and the sum
- * of the event-measured durations. Index: 0 decode attention, 1 LSE merge,
- * 2 append copy, 3 inspection gather. */
+ * While profiling is on, the library's launches on the tree's stream are
+ * bracketed by pairs of CUDA events (the attention kernels of one call
+ * together). tp_profile_stop waits for the stream and returns, per kernel
+ * kind, the number of kernels launched and the sum of the event-measured
+ * durations of their brackets. Index: 0 attention (decode and prefill; the
+ * decode schedule's patch kernel is counted here, untimed), 1 LSE merge,
+ * 2 appends (copies, stand-in activations, the rollout's token steps),
+ * 3 inspection gather. tp_decode_noalloc and tp_tree_advantage are not
+ * profiled. */
 #define TP_KERNEL_KINDS 4
 typedef struct {
     int64_t launches[TP_KERNEL_KINDS];

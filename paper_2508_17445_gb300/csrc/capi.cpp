@@ -218,6 +218,7 @@ tp_status patch_cached_schedule(tp_tree* t) {
     st = stage_upload(t, t->d_patch, t->patch_words.data(), 2 * (int64_t)n);
     if (st != TP_OK) return st;
     cudaError_t e = tp::launch_patch(t->d_sched, t->d_patch, n, t->stream);
+    tp::count_kernels(t, tp::KK_DECODE, 1);
     if (e != cudaSuccess) return cuda_fail(t, e, "schedule patch kernel");
     return TP_OK;
 }
@@ -243,10 +244,17 @@ LaunchTimer::LaunchTimer(tp_tree* t, int kind) : t_(t), kind_(kind) {
         return;
     }
     cudaEventRecord(a, t_->stream);
-    t_->timed.push_back({kind_, a, b_});
+    index_ = t_->timed.size();
+    t_->timed.push_back({kind_, a, b_, 1});
 }
 LaunchTimer::~LaunchTimer() {
     if (b_) cudaEventRecord(b_, t_->stream);
+}
+void LaunchTimer::kernels(int n) {
+    if (b_) t_->timed[index_].kernels = n;
+}
+void count_kernels(tp_tree* t, int kind, int n) {
+    if (t->profiling) t->untimed[kind] += n;
 }
 }  // namespace tp
 
@@ -464,6 +472,7 @@ tp_status tp_synth_tokens(tp_tree* t, uint64_t seed, tp_node node, int32_t pos0,
     a.q_width = t->cfg.num_q_heads * t->cfg.head_dim;
     a.node0 = node;
     a.pos0 = pos0;
+    tp::LaunchTimer timer(t, tp::KK_APPEND);
     cudaError_t e = tp::launch_synth(a, t->stream);
     if (e != cudaSuccess) return cuda_fail(t, e, "synth kernel");
     return TP_OK;
@@ -754,6 +763,7 @@ tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O
     if (a.n_units > 0) {
         tp::LaunchTimer timer(t, tp::KK_DECODE);
         e = tp::launch_decode(hd, a, t->stream, t->side, t->ev_fork, t->ev_join);
+        timer.kernels((S.n_tc > 0) + (S.n_tensor > 0) + (S.n_units > S.n_tc + S.n_tensor));
     }
     if (e != cudaSuccess) return cuda_fail(t, e, "decode kernel");
 
@@ -857,6 +867,7 @@ tp_status tp_profile_start(tp_tree* t) {
     if (e != cudaSuccess) return cuda_fail(t, e, "cudaStreamSynchronize");
     t->timed.clear();
     t->ev_used = 0;
+    for (int64_t& k : t->untimed) k = 0;
     t->profiling = true;
     return TP_OK;
 }
@@ -872,8 +883,12 @@ tp_status tp_profile_stop(tp_tree* t, tp_kernel_times* out) {
         float ms = 0.f;
         e = cudaEventElapsedTime(&ms, x.a, x.b);
         if (e != cudaSuccess) return cuda_fail(t, e, "cudaEventElapsedTime");
-        out->launches[x.kind] += 1;
+        out->launches[x.kind] += x.kernels;
         out->milliseconds[x.kind] += ms;
+    }
+    for (int k = 0; k < TP_KERNEL_KINDS; ++k) {
+        out->launches[k] += t->untimed[k];
+        t->untimed[k] = 0;
     }
     t->timed.clear();
     t->ev_used = 0;

@@ -298,9 +298,11 @@ struct tp_tree {
     struct Timed {
         int kind;
         cudaEvent_t a, b;
+        int kernels;  // kernels launched inside the bracket
     };
     std::vector<Timed> timed;
     size_t ev_used = 0;
+    int64_t untimed[4] = {0, 0, 0, 0};  // kernels counted without their own events, per kind
 
     // schedule cache: the device copy of the last uploaded schedule
     tp::Schedule sched;
@@ -326,12 +328,16 @@ class LaunchTimer {
    public:
     LaunchTimer(tp_tree* t, int kind);
     ~LaunchTimer();
+    void kernels(int n);  // the bracket launched n kernels (default 1)
 
    private:
     tp_tree* t_;
     int kind_;
     cudaEvent_t b_ = nullptr;
+    size_t index_ = 0;
 };
+// Counts n kernels of a kind while profiling, without timing them.
+void count_kernels(tp_tree* t, int kind, int n);
 
 // capi.cpp
 tp_status cuda_fail(tp_tree* t, cudaError_t e, const char* what);

@@ -177,7 +177,11 @@ class Rollout {
         a.q_width = t_->cfg.num_q_heads * t_->cfg.head_dim;
         a.node0 = node;
         a.pos0 = t_->nodes[(size_t)node].n_tokens;
-        cudaError_t e = tp::launch_synth(a, t_->stream);
+        cudaError_t e;
+        {
+            tp::LaunchTimer timer(t_, tp::KK_APPEND);
+            e = tp::launch_synth(a, t_->stream);
+        }
         if (e != cudaSuccess) return tp::cuda_fail(t_, e, "synth kernel");
         return tp_append_segment(t_, node, n, k_.p, v_.p);
     }

@@ -303,16 +303,22 @@ def test_schedule_cache_follows_tree_changes():
     f.close()
 
 
-def test_profile_counts_launches():
+@pytest.mark.parametrize("flags", [0, tp.TP_MMA_SYNC, tp.TP_DECODE_CUDA_CORE_SMALL])
+def test_profile_counts_kernel_launches(flags):
     s = workloads.tiny()
     f, ids = build_forest(s)
     leaves = [ids[x] for x in s.leaves]
+    d = tp.tp_debug_schedule(f.handle, leaves, flags)
+    n_units, n_tc, n_mma = len(d["units"]), d["n_tc_units"], d["n_tensor_units"]
+    per_call = (n_tc > 0) + (n_mma > 0) + (n_units > n_tc + n_mma)  # attention kernels of one call
+    assert per_call >= 1
     Q = s.q(DEV)
+    f.decode(leaves, Q, flags=flags)  # builds and caches the schedule
     tp.tp_profile_start(f.handle)
     for _ in range(3):
-        f.decode(leaves, Q)
+        f.decode(leaves, Q, flags=flags)
     t = tp.tp_profile_stop(f.handle)
-    assert t["decode"]["launches"] == 3 and t["merge"]["launches"] == 3
+    assert t["decode"]["launches"] == 3 * per_call and t["merge"]["launches"] == 3
     assert t["decode"]["ms"] > 0
     f.sync()
     f.close()
