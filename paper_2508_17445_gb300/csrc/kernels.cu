@@ -1875,10 +1875,11 @@ __global__ void __launch_bounds__(kTcThreads, 2) decode_tc_kernel(const DecodeAr
         tc_consume<HD, CAUSAL>(a, ctl);
     else if (warp == kTcStreamerWarp) {
         if ((tid & 31) == 0) tc_stream<HD>(a, ctl, ring);
-    } else if (warp == kTcFetcherWarp)
+    } else if (warp == kTcFetcherWarp) {
         tc_fetch<HD>(a, ctl, qbuf);
-    else if ((tid & 31) == 0)
-        tc_issue<HD>(a, ctl, ring, qbuf);
+    } else if (warp == kTcIssuerWarp) {
+        if ((tid & 31) == 0) tc_issue<HD>(a, ctl, ring, qbuf);
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
