@@ -349,3 +349,20 @@ def test_full_size_sampled(name, k):
         check(O, LSE, o_ref, lse_ref, a_ref, rows=rows)
         assert torch.isfinite(O.float()).all() and torch.isfinite(LSE).all()
     f.close()
+
+
+# --------------------------------------------------------------------------
+# randomized sweep: more seeds, head shapes and routing flags
+# --------------------------------------------------------------------------
+SWEEP_HEADS = [workloads.Heads(4, 1, 64), workloads.Heads(8, 2, 64), workloads.Heads(28, 4, 128),
+               workloads.Heads(64, 8, 128), workloads.Heads(16, 16, 128), workloads.Heads(32, 2, 64)]
+
+
+@pytest.mark.parametrize("seed", range(100, 124))
+def test_random_forest_sweep(seed):
+    rng = np.random.default_rng(seed)
+    heads = SWEEP_HEADS[seed % len(SWEEP_HEADS)]
+    s = workloads.random_tree(seed=seed, heads=heads, n_prompts=int(rng.integers(1, 5)),
+                              max_depth=int(rng.integers(1, 7)), prompt_range=(1, int(rng.integers(2, 700))),
+                              seg_range=(1, int(rng.integers(2, 300))), max_kids=int(rng.integers(1, 5)))
+    run_and_compare(s, flags=FLAG_SETS[(seed // len(SWEEP_HEADS)) % len(FLAG_SETS)])

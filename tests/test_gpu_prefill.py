@@ -138,3 +138,20 @@ def test_prefill_last_token_matches_decode():
     assert (O1.float() - O2.float()).abs().max().item() <= 2 ** -7
     assert (L1 - L2).abs().max().item() <= 5e-5
     f.close()
+
+
+@pytest.mark.parametrize("seed", range(100, 112))
+def test_prefill_random_sweep(seed):
+    rng = np.random.default_rng(seed)
+    heads = [workloads.Heads(8, 2, 64), workloads.Heads(28, 4, 128), workloads.Heads(64, 8, 128),
+             workloads.Heads(16, 16, 128)][seed % 4]
+    s = workloads.random_tree(seed=seed, n_prompts=int(rng.integers(1, 4)), max_depth=int(rng.integers(1, 6)),
+                              heads=heads, prompt_range=(1, int(rng.integers(2, 600))),
+                              seg_range=(1, int(rng.integers(2, 300))))
+    model = oracle.OracleForest(block_tokens=32).replay(s)
+    live = [x for x in model.nodes if model.nodes[x].state != "dead" and model.nodes[x].n_tokens > 0]
+    pick = [live[int(i)] for i in rng.integers(0, len(live), min(len(live), 10))]
+    counts = [int(rng.integers(0, model.nodes[x].n_tokens + 1)) for x in pick]
+    if sum(counts) == 0:
+        counts[0] = 1
+    run_prefill(s, pick, counts, seed=seed, flags=FLAGS[seed % 2])
