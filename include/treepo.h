@@ -258,6 +258,15 @@ tp_status tp_decode_host(tp_tree* tree, const tp_node* leaves, int32_t n, const 
 tp_status tp_prefill_host(tp_tree* tree, const tp_node* nodes, const int32_t* n_queries, int32_t n,
                           const void* Q_host, void* O_host, float* LSE_host, uint32_t flags);
 
+/* Failure-reporting probe (testing; no counterpart in the paper). Launches,
+ * on the tree's stream, one small kernel that runs the attention kernels'
+ * bounded wait on a barrier nothing ever completes, with a limit of limit_ns
+ * (1e3 .. 1e9) instead of their 2 s; when it runs out the kernel sets the
+ * device error flag and returns, so the next tp_sync returns TP_ERR_DEVICE
+ * and the tree stays usable. No fault and no trap is involved. Errors:
+ * TP_ERR_INVALID_ARG (limit out of range, metadata-only tree), TP_ERR_CUDA. */
+tp_status tp_debug_wait_probe(tp_tree* tree, int64_t limit_ns);
+
 /* Wait for the tree's stream (and the copy streams of the host-buffer
  * calls); TP_ERR_DEVICE if a kernel gave up a bounded wait since the last
  * tp_sync (the flag is then cleared), TP_ERR_CUDA on a CUDA error. */

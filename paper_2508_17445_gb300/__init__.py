@@ -24,7 +24,7 @@ __all__ = [
     "tp_sync", "tp_last_error", "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop",
     "tp_debug_path", "tp_debug_gather",
     "tp_debug_schedule", "tp_decode_noalloc", "tp_append_tokens", "tp_synth_tokens", "tp_branch_assign",
-    "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "tp_prefill", "tp_debug_prefill_schedule", "tp_decode_host", "tp_prefill_host", "TpRolloutParams", "TpRolloutStats",
+    "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "tp_prefill", "tp_debug_prefill_schedule", "tp_decode_host", "tp_prefill_host", "tp_debug_wait_probe", "TpRolloutParams", "TpRolloutStats",
     "TpRolloutProbe", "rollout_params", "TP_BRANCH_EVEN", "TP_BRANCH_LOGP_HIGH", "TP_BRANCH_LOGP_LOW",
     "EVENT_NAMES", "TP_SEG_EOS", "TP_SEG_BOXED", "TP_SEG_FAILED", "TP_SEG_MAX_DEPTH", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE", "TP_DECODE_TCGEN05", "TP_DECODE_ALL_TCGEN05", "TP_MMA_SYNC",
     "EXPORTED_SYMBOLS",
@@ -56,7 +56,7 @@ EXPORTED_SYMBOLS = (
     "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop", "tp_debug_path",
     "tp_debug_gather", "tp_debug_schedule", "tp_decode_noalloc", "tp_append_tokens", "tp_synth_tokens",
     "tp_branch_assign", "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "tp_prefill",
-    "tp_debug_prefill_schedule", "tp_decode_host", "tp_prefill_host",
+    "tp_debug_prefill_schedule", "tp_decode_host", "tp_prefill_host", "tp_debug_wait_probe",
 )
 
 
@@ -155,6 +155,7 @@ def load_library() -> ctypes.CDLL:
         "tp_prefill": (I32, [P, P, P, I32, P, P, P, U32]),
         "tp_decode_host": (I32, [P, P, I32, P, P, P, U32]),
         "tp_prefill_host": (I32, [P, P, P, I32, P, P, P, U32]),
+        "tp_debug_wait_probe": (I32, [P, I64]),
         "tp_debug_prefill_schedule": (I32, [P, P, P, I32, U32, P, I64, P]),
     }
     for name, (res, args) in sig.items():
@@ -316,6 +317,11 @@ def tp_prefill_host(h, nodes: Sequence[int], n_queries: Sequence[int], Q, O, LSE
     _check(h, load_library().tp_prefill_host(h, arr.ctypes.data if len(arr) else None,
                                              m.ctypes.data if len(m) else None, len(arr), _host_ptr(Q),
                                              _host_ptr(O), _host_ptr(LSE), flags))
+
+
+def tp_debug_wait_probe(h, limit_ns: int) -> None:
+    """Launch the bounded-wait probe: the next tp_sync raises TreepoError DEVICE."""
+    _check(h, load_library().tp_debug_wait_probe(h, int(limit_ns)))
 
 
 def _parse_schedule(w: np.ndarray) -> Dict[str, np.ndarray]:

@@ -895,6 +895,15 @@ tp_status tp_profile_stop(tp_tree* t, tp_kernel_times* out) {
     return TP_OK;
 }
 
+tp_status tp_debug_wait_probe(tp_tree* t, int64_t limit_ns) {
+    if (!t) return TP_ERR_INVALID_ARG;
+    if (!t->cfg.pool) return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree launches no kernels");
+    if (limit_ns < 1000 || limit_ns > 1000000000) return fail(t, TP_ERR_INVALID_ARG, "limit_ns must lie in [1e3, 1e9]");
+    cudaError_t e = tp::launch_wait_probe(t->d_err, (uint64_t)limit_ns, t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "wait probe kernel");
+    return TP_OK;
+}
+
 tp_status tp_sync(tp_tree* t) {
     if (!t) return TP_ERR_INVALID_ARG;
     if (!t->cfg.pool) return TP_OK;

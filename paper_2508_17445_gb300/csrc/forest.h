@@ -177,6 +177,7 @@ cudaError_t launch_merge(int head_dim, const MergeArgs& a, cudaStream_t s);
 cudaError_t launch_gather(int head_dim, const GatherArgs& a, int64_t n_tokens, cudaStream_t s);
 // sched[pairs[2k]] = pairs[2k + 1] for k < n.
 cudaError_t launch_patch(int32_t* sched, const int32_t* pairs, int32_t n, cudaStream_t s);
+cudaError_t launch_wait_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s);
 cudaError_t launch_append_tokens(int head_dim, const AppendTokensArgs& a, cudaStream_t s);
 cudaError_t launch_synth(const SynthArgs& a, cudaStream_t s);
 cudaError_t launch_rollout_step(int head_dim, const StepArgs& a, cudaStream_t s);

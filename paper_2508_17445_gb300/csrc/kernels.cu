@@ -95,12 +95,12 @@ __device__ __forceinline__ uint64_t global_ns() {
 }
 
 // Wait for an mbarrier phase with a time limit; false if the limit ran out.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint64_t limit_ns = kWaitLimitNs) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_ns();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
-        if ((i & 63) == 0 && global_ns() - t0 > kWaitLimitNs) return false;
+        if ((i & 63) == 0 && global_ns() - t0 > limit_ns) return false;
     }
 }
 
@@ -2096,6 +2096,24 @@ cudaError_t noalloc_scratch(void** device_ptr) {
     }
     *device_ptr = addr[dev];
     return cudaSuccess;
+}
+
+// Failure-reporting probe: the attention kernels' bounded wait, on a barrier
+// nothing ever completes and with a short limit; when it runs out the kernel
+// sets its bit of the device error flag and returns, as they do.
+__global__ void wait_probe_kernel(int32_t* err, uint64_t limit_ns) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && !mbar_wait(smem_u32(&bar), 0, limit_ns)) atomicOr(err, 32);
+}
+
+cudaError_t launch_wait_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s) {
+    wait_probe_kernel<<<1, 32, 0, s>>>(err, limit_ns);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_patch(int32_t* sched, const int32_t* pairs, int32_t n, cudaStream_t s) {

@@ -303,6 +303,31 @@ def test_schedule_cache_follows_tree_changes():
     f.close()
 
 
+def test_bounded_wait_reports_and_the_tree_stays_usable():
+    # a kernel whose bounded wait (the attention kernels' helper, 20 ms limit
+    # instead of 2 s) runs out on a barrier nothing completes: tp_sync reports
+    # it, clears the flag, and the same tree decodes bit-identically afterwards
+    s = workloads.tiny(seed=1)
+    f, ids = build_forest(s)
+    leaves = [ids[x] for x in s.leaves]
+    Q = s.q(DEV)
+    O1, L1 = f.decode(leaves, Q)
+    f.sync()
+    O1, L1 = O1.clone(), L1.clone()
+    with pytest.raises(tp.TreepoError) as e:
+        tp.tp_debug_wait_probe(f.handle, 10)  # below the 1 us floor
+    assert e.value.code == "INVALID_ARG"
+    tp.tp_debug_wait_probe(f.handle, 20_000_000)
+    with pytest.raises(tp.TreepoError) as e:
+        f.sync()
+    assert e.value.code == "DEVICE"
+    f.sync()  # the flag was cleared
+    O2, L2 = f.decode(leaves, Q)
+    f.sync()
+    assert torch.equal(O1.view(torch.int16), O2.view(torch.int16)) and torch.equal(L1, L2)
+    f.close()
+
+
 @pytest.mark.parametrize("flags", [0, tp.TP_MMA_SYNC, tp.TP_DECODE_CUDA_CORE_SMALL])
 def test_profile_counts_kernel_launches(flags):
     s = workloads.tiny()

@@ -231,6 +231,13 @@ class _FakePtr:
         return 0x1000
 
 
+def test_wait_probe_needs_a_device_tree():
+    f = meta_forest(pool_blocks=4)
+    with pytest.raises(tp.TreepoError) as e:
+        tp.tp_debug_wait_probe(f.handle, 1_000_000)
+    assert e.value.code == "INVALID_ARG"
+
+
 def test_host_buffer_calls_check_their_arguments():
     import torch
     f = meta_forest(pool_blocks=8)
