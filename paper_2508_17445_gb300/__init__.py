@@ -500,6 +500,32 @@ class Forest:
         tp_decode_ex(self.handle, leaves, Q, O, LSE, flags)
         return O, LSE
 
+    def decode_host(self, leaves: Sequence[int], Q, flags: int = 0, out=None):
+        """decode with host Q (CPU tensor, ideally pinned); O and LSE are
+        pinned host tensors, valid after sync()."""
+        import torch
+        n, hq, hd = Q.shape
+        if out is None:
+            O = torch.empty((n, hq, hd), dtype=torch.bfloat16).pin_memory()
+            LSE = torch.empty((n, hq), dtype=torch.float32).pin_memory()
+        else:
+            O, LSE = out
+        tp_decode_host(self.handle, leaves, Q, O, LSE, flags)
+        return O, LSE
+
+    def prefill(self, nodes: Sequence[int], n_queries: Sequence[int], Q, flags: int = 0, out=None):
+        """Causal attention of the last n_queries[i] tokens of nodes[i] over
+        their paths; Q: [sum n_queries][Hq][hd] on the device."""
+        import torch
+        n, hq, hd = Q.shape
+        if out is None:
+            O = torch.empty((n, hq, hd), dtype=torch.bfloat16, device=Q.device)
+            LSE = torch.empty((n, hq), dtype=torch.float32, device=Q.device)
+        else:
+            O, LSE = out
+        tp_prefill(self.handle, nodes, n_queries, Q, O, LSE, flags)
+        return O, LSE
+
     def append_tokens(self, nodes: Sequence[int], K=None, V=None) -> None:
         tp_append_tokens(self.handle, nodes, K, V)
 

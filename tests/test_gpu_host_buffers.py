@@ -160,3 +160,22 @@ def test_host_prefill_equals_device_prefill(flags):
     for (o, lse), (o_ref, lse_ref) in zip(outs, refs):
         assert _same(o, o_ref) and _same(lse, lse_ref)
     f.close()
+
+
+def test_forest_wrappers():
+    s = workloads.segment_prefill(seed=7, n_prompts=1, prompt_len=200, fanout=2, seg_len=40)
+    f, ids = _forest(s)
+    leaves = [ids[x] for x in s.leaves]
+    q = _queries(len(leaves), s.heads, 60)
+    O, L = f.decode(leaves, q.to(DEV))
+    Oh, Lh = f.decode_host(leaves, q)
+    f.sync()
+    assert _same(Oh, O.cpu()) and _same(Lh, L.cpu())
+    q16 = _queries(16, s.heads, 61).to(DEV)
+    O2, L2 = f.prefill([leaves[0]], [16], q16)
+    O3 = torch.empty_like(q16)
+    L3 = torch.empty(16, s.heads.num_q_heads, dtype=torch.float32, device=DEV)
+    tp.tp_prefill(f.handle, [leaves[0]], [16], q16, O3, L3)
+    f.sync()
+    assert _same(O2.cpu(), O3.cpu()) and _same(L2.cpu(), L3.cpu())
+    f.close()
