@@ -111,6 +111,56 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
         : "memory");
 }
 
+// L2 residency: a decode call streams GBs of K/V through the 129 MB L2 once,
+// while its fp32 partials (tens of MB) are written by the attention kernels
+// and read back by the merge. K/V copies read once go in as evict-first, the
+// partials as evict-last, and the merge reads them as evict-first (dead
+// after), so they are served from L2 instead of a round trip through HBM.
+__device__ __forceinline__ uint64_t l2_evict_first() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+
+__device__ __forceinline__ uint64_t l2_evict_last() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+
+__device__ __forceinline__ void bulk_g2s_hint(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar,
+                                              uint64_t pol) {
+    asm volatile(
+        "cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+            dst),
+        "l"(src), "r"(bytes), "r"(bar), "l"(pol)
+        : "memory");
+}
+
+__device__ __forceinline__ void st_f2_hint(float* p, float x, float y, uint64_t pol) {
+    asm volatile("st.global.L2::cache_hint.v2.f32 [%0], {%1, %2}, %3;" ::"l"(p), "f"(x), "f"(y), "l"(pol) : "memory");
+}
+
+__device__ __forceinline__ void st_f4_hint(float* p, float4 v, uint64_t pol) {
+    asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(p), "f"(v.x), "f"(v.y), "f"(v.z),
+                 "f"(v.w), "l"(pol)
+                 : "memory");
+}
+
+__device__ __forceinline__ float4 ld_f4_hint(const float* p, uint64_t pol) {
+    float4 v;
+    asm volatile("ld.global.L2::cache_hint.v4.f32 {%0, %1, %2, %3}, [%4], %5;"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "l"(p), "l"(pol));
+    return v;
+}
+
+__device__ __forceinline__ float2 ld_f2_hint(const float* p, uint64_t pol) {
+    float2 v;
+    asm volatile("ld.global.L2::cache_hint.v2.f32 {%0, %1}, [%2], %3;" : "=f"(v.x), "=f"(v.y) : "l"(p), "l"(pol));
+    return v;
+}
+
 // 16-byte global -> shared copy that bypasses registers (cp.async)
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
@@ -150,6 +200,13 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 __device__ __forceinline__ void st_global_v8(void* dst, const uint32_t* w) {
     asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(dst), "r"(w[0]), "r"(w[1]),
                  "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                 : "memory");
+}
+
+// the same with an L2 cache policy
+__device__ __forceinline__ void st_global_v8_hint(void* dst, const uint32_t* w, uint64_t pol) {
+    asm volatile("st.global.L2::cache_hint.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8}, %9;" ::"l"(dst), "r"(w[0]),
+                 "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7]), "l"(pol)
                  : "memory");
 }
 
@@ -558,8 +615,14 @@ __device__ __forceinline__ void issue_pair(const DecodeArgs& a, CtlT& c, int kvh
 #pragma unroll
         for (int h = 0; h < HD / 64; ++h) {
             const int so = h * kBlockTokens * 128, dofs = h * kStageTokens * 128 + j * kBlockTokens * 128;
-            bulk_g2s(smem_u32(sk + dofs), src + so, valid[j] * 128, bar);
-            bulk_g2s(smem_u32(sv + dofs), src + (int64_t)a.hkv * a.head_bytes + so, valid[j] * 128, bar);
+            if (a.vis) {  // prefill: the query blocks of a path re-read its K/V from L2
+                bulk_g2s(smem_u32(sk + dofs), src + so, valid[j] * 128, bar);
+                bulk_g2s(smem_u32(sv + dofs), src + (int64_t)a.hkv * a.head_bytes + so, valid[j] * 128, bar);
+            } else {
+                const uint64_t pol = l2_evict_first();
+                bulk_g2s_hint(smem_u32(sk + dofs), src + so, valid[j] * 128, bar, pol);
+                bulk_g2s_hint(smem_u32(sv + dofs), src + (int64_t)a.hkv * a.head_bytes + so, valid[j] * 128, bar, pol);
+            }
         }
     }
 }
@@ -823,6 +886,7 @@ struct CudaCorePath {
             const int qh = u.kvh * a.group + item_row % a.group;
             float* dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
             const float inv = 1.f / L;
+            const uint64_t pol = l2_evict_last();
             for (int d = q4 * 4; d < HD; d += 16) {
                 float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
                 for (int s = 0; s < n_sp; ++s) {
@@ -832,7 +896,7 @@ struct CudaCorePath {
                     acc.z += w[s] * x.z;
                     acc.w += w[s] * x.w;
                 }
-                *reinterpret_cast<float4*>(dst + d) = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+                st_f4_hint(dst + d, make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv), pol);
             }
             if (q4 == 0) a.part_lse[(int64_t)slot * a.hq + qh] = M + __log2f(L);
         }
@@ -1037,9 +1101,9 @@ struct TensorPath {
             }
             const int slot = u.slot_base + item_row / a.group;
             float* dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
+            const uint64_t pol = l2_evict_last();
 #pragma unroll
-            for (int j = 0; j < NT; ++j)
-                *reinterpret_cast<float2*>(dst + j * 8 + 2 * c4) = make_float2(o[j][2 * h] * inv, o[j][2 * h + 1] * inv);
+            for (int j = 0; j < NT; ++j) st_f2_hint(dst + j * 8 + 2 * c4, o[j][2 * h] * inv, o[j][2 * h + 1] * inv, pol);
             if (c4 == 0) a.part_lse[(int64_t)slot * a.hq + qh] = m_run[h] + __log2f(l_run[h]);
         }
     }
@@ -1783,6 +1847,7 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
             }
         }
         const float inv = 1.f / l;
+        const uint64_t pol = l2_evict_last();
         // 32-byte stores (a full sector per lane) where the rows allow them:
         // the partial buffer always, the caller's O when its base is 32-byte
         // aligned (rows are multiples of 256 bytes, so the base decides)
@@ -1816,7 +1881,7 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
                         uint32_t w[8];
 #pragma unroll
                         for (int e = 0; e < 8; ++e) w[e] = __float_as_uint(__uint_as_float(ov[h][t + e]) * inv);
-                        st_global_v8(dst + c0 + t, w);
+                        st_global_v8_hint(dst + c0 + t, w, pol);
                     }
                 }
             }
@@ -1901,6 +1966,7 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
 #pragma unroll
     for (int d = 0; d < DPL; ++d) acc[d] = 0.f;
     float M = -INFINITY, L = 0.f;
+    const uint64_t pol = l2_evict_first();  // each partial row is read once
     // slots in chunks of 32: lane k fetches slot k's index and LSE, then the
     // warp folds the chunk's partial rows, four loads in flight per lane
     for (int c0 = 0; c0 < ns; c0 += 32) {
@@ -1936,10 +2002,10 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
                 wj[u] = __shfl_sync(0xffffffffu, w, j + u);
                 const float* src = a.part_o + (sl * a.hq + qh) * HD + lane * DPL;
                 if constexpr (DPL == 4) {
-                    const float4 v = *reinterpret_cast<const float4*>(src);
+                    const float4 v = ld_f4_hint(src, pol);
                     x[u][0] = v.x, x[u][1] = v.y, x[u][2] = v.z, x[u][3] = v.w;
                 } else {
-                    const float2 v = *reinterpret_cast<const float2*>(src);
+                    const float2 v = ld_f2_hint(src, pol);
                     x[u][0] = v.x, x[u][1] = v.y;
                 }
             }
@@ -1952,8 +2018,16 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
             const int64_t sl = __shfl_sync(0xffffffffu, slot, j);
             const float wj = __shfl_sync(0xffffffffu, w, j);
             const float* src = a.part_o + (sl * a.hq + qh) * HD + lane * DPL;
+            float xs[DPL];
+            if constexpr (DPL == 4) {
+                const float4 v = ld_f4_hint(src, pol);
+                xs[0] = v.x, xs[1] = v.y, xs[2] = v.z, xs[3] = v.w;
+            } else {
+                const float2 v = ld_f2_hint(src, pol);
+                xs[0] = v.x, xs[1] = v.y;
+            }
 #pragma unroll
-            for (int d = 0; d < DPL; ++d) acc[d] += wj * src[d];
+            for (int d = 0; d < DPL; ++d) acc[d] += wj * xs[d];
         }
     }
     const float inv = 1.f / L;
