@@ -753,6 +753,7 @@ tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O
     a.hkv = t->cfg.num_kv_heads;
     a.group = hq / t->cfg.num_kv_heads;
     a.qk_scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
+    a.kv_read_once = S.kv_read_once ? 1 : 0;
     cudaError_t e = cudaSuccess;
     if (S.n_tc > 0 && S.n_units > S.n_tc && !t->side) {  // concurrent tcgen05 units need a second stream
         e = cudaStreamCreateWithFlags(&t->side, cudaStreamNonBlocking);
@@ -839,6 +840,7 @@ tp_status tp_decode_noalloc(tp_tree* t, const tp_node* leaves, int32_t n, const 
     a.hkv = t->cfg.num_kv_heads;
     a.group = hq / t->cfg.num_kv_heads;
     a.qk_scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
+    a.kv_read_once = S.kv_read_once ? 1 : 0;
     e = tp::launch_decode(hd, a, t->stream);
     if (e != cudaSuccess) return cuda_fail(t, e, "decode kernel");
     tp::MergeArgs m;

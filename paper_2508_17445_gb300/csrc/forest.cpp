@@ -374,6 +374,11 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
         S.leaf_tail[2 * k + 1] = (int32_t)S.off_tiles + X.tail_tile[k];
     }
     S.prefill = false;
+    // With the default routing the mma.sync / CUDA-core kernel (the only one
+    // that uses this) gets single-leaf groups of at most 16 rows, one unit per
+    // (block, kv head); the no-share control and the other routings give it
+    // units that read the same blocks.
+    S.kv_read_once = !(flags & (TP_DECODE_NO_SHARE | TP_DECODE_TCGEN05 | TP_MMA_SYNC));
     S.off_unit_pos = S.off_vis = 0;
     return TP_OK;
 }
@@ -468,6 +473,7 @@ tp_status build_prefill_schedule(tp_tree* t, const tp_node* nodes, const int32_t
     merge_csr(X, (int32_t)n_q);
 
     S.prefill = true;
+    S.kv_read_once = false;  // the query blocks of a path re-read its K/V
     S.n_units = (int32_t)(recs.size() / W);
     S.n_tc = use_tc ? S.n_units : 0;
     S.n_tensor = use_tc ? 0 : S.n_units;

@@ -71,6 +71,7 @@ struct DecodeArgs {
     int32_t hkv;
     int32_t group;
     float qk_scale_log2;  // log2(e) / sqrt(hd)
+    int32_t kv_read_once = 0;  // the mma.sync kernel's units read disjoint K/V: copy them in as L2 evict-first
 };
 
 struct MergeArgs {
@@ -218,6 +219,7 @@ struct Schedule {
     int32_t n_units = 0, n_tiles = 0, n_occ = 0, n = 0, n_slots = 0, n_merge = 0, n_tensor = 0, n_tc = 0;
     int64_t off_units = 0, off_tiles = 0, off_occ = 0, off_merge_off = 0, off_merge_slot = 0;
     bool prefill = false;
+    bool kv_read_once = false;  // see DecodeArgs::kv_read_once
     int64_t off_unit_pos = 0, off_vis = 0;
     // (leaf node, word index of the last tile of that leaf) for every place a
     // listed leaf's last block appears: appends that stay inside that block

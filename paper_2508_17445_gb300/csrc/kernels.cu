@@ -615,7 +615,7 @@ __device__ __forceinline__ void issue_pair(const DecodeArgs& a, CtlT& c, int kvh
 #pragma unroll
         for (int h = 0; h < HD / 64; ++h) {
             const int so = h * kBlockTokens * 128, dofs = h * kStageTokens * 128 + j * kBlockTokens * 128;
-            if (a.vis) {  // prefill: the query blocks of a path re-read its K/V from L2
+            if (!a.kv_read_once) {  // blocks re-read by other units (prefill, no-share control): keep them in L2
                 bulk_g2s(smem_u32(sk + dofs), src + so, valid[j] * 128, bar);
                 bulk_g2s(smem_u32(sv + dofs), src + (int64_t)a.hkv * a.head_bytes + so, valid[j] * 128, bar);
             } else {
