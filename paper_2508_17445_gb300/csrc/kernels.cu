@@ -155,6 +155,13 @@ __device__ __forceinline__ float4 ld_f4_hint(const float* p, uint64_t pol) {
     return v;
 }
 
+// Drop a 128-byte L2 line without writing it back (its contents become
+// undefined): for partial rows the merge has consumed.
+__device__ __forceinline__ void l2_discard(const void* p) {
+    if ((reinterpret_cast<uintptr_t>(p) & 127) == 0)  // whole lines only (the partial rows are 256-byte aligned)
+        asm volatile("discard.global.L2 [%0], 128;" ::"l"(p) : "memory");
+}
+
 __device__ __forceinline__ float2 ld_f2_hint(const float* p, uint64_t pol) {
     float2 v;
     asm volatile("ld.global.L2::cache_hint.v2.f32 {%0, %1}, [%2], %3;" : "=f"(v.x), "=f"(v.y) : "l"(p), "l"(pol));
@@ -1992,15 +1999,23 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
         for (int off = 16; off; off >>= 1) ws += __shfl_xor_sync(0xffffffffu, ws, off);
         L += ws;
         const int cnt = min(32, ns - c0);
+        // A partial row is read by this warp only (slots are per leaf
+        // occurrence): once folded, its lines are dropped from L2 instead of
+        // being written back to HBM. Each 128-byte line is dropped by the
+        // first lane that read from it, after the warp has used the loads.
+        constexpr int kLanesPerLine = 128 / (DPL * 4);
+        const bool line_lead = (lane & (kLanesPerLine - 1)) == 0;
         int j = 0;
         for (; j + 4 <= cnt; j += 4) {
             float wj[4];
             float x[4][DPL];
+            const float* srcs[4];
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int64_t sl = __shfl_sync(0xffffffffu, slot, j + u);
                 wj[u] = __shfl_sync(0xffffffffu, w, j + u);
                 const float* src = a.part_o + (sl * a.hq + qh) * HD + lane * DPL;
+                srcs[u] = src;
                 if constexpr (DPL == 4) {
                     const float4 v = ld_f4_hint(src, pol);
                     x[u][0] = v.x, x[u][1] = v.y, x[u][2] = v.z, x[u][3] = v.w;
@@ -2013,6 +2028,10 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
             for (int u = 0; u < 4; ++u)
 #pragma unroll
                 for (int d = 0; d < DPL; ++d) acc[d] += wj[u] * x[u][d];
+            __syncwarp();
+            if (line_lead)
+#pragma unroll
+                for (int u = 0; u < 4; ++u) l2_discard(srcs[u]);
         }
         for (; j < cnt; ++j) {
             const int64_t sl = __shfl_sync(0xffffffffu, slot, j);
@@ -2028,6 +2047,8 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
             }
 #pragma unroll
             for (int d = 0; d < DPL; ++d) acc[d] += wj * xs[d];
+            __syncwarp();
+            if (line_lead) l2_discard(src);
         }
     }
     const float inv = 1.f / L;
