@@ -71,7 +71,9 @@ struct DecodeArgs {
     int32_t hkv;
     int32_t group;
     float qk_scale_log2;  // log2(e) / sqrt(hd)
-    int32_t kv_read_once = 0;  // the mma.sync kernel's units read disjoint K/V: copy them in as L2 evict-first
+    int32_t kv_read_once = 0;  // decode, default routing: the mma.sync kernel's units, and the tcgen05
+                               // units of single-row-block items, read disjoint K/V (copied in as L2
+                               // evict-first)
 };
 
 struct MergeArgs {

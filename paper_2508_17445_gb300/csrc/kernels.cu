@@ -1511,7 +1511,7 @@ __device__ void tc_fetch(const DecodeArgs& a, CtlTc& c, uint8_t* qbuf) {
 // missing second tile.
 template <int HD>
 __device__ __forceinline__ void issue_half(const DecodeArgs& a, int kvh, int kv, uint8_t* dst, const int32_t (&w)[2],
-                                           uint32_t bar) {
+                                           uint32_t bar, bool once) {
     uint32_t bytes = 0;
     int valid[2] = {0, 0};
     for (int j = 0; j < 2; ++j)
@@ -1525,9 +1525,13 @@ __device__ __forceinline__ void issue_half(const DecodeArgs& a, int kvh, int kv,
         const uint8_t* src = a.pool + (int64_t)(w[j] >> kTileValidBits) * a.block_bytes +
                              (int64_t)(kv * a.hkv + kvh) * a.head_bytes;
 #pragma unroll
-        for (int h = 0; h < HD / 64; ++h)
-            bulk_g2s(smem_u32(dst + h * kStageTokens * 128 + j * kBlockTokens * 128), src + h * kBlockTokens * 128,
-                     valid[j] * 128, bar);
+        for (int h = 0; h < HD / 64; ++h) {
+            const uint32_t d = smem_u32(dst + h * kStageTokens * 128 + j * kBlockTokens * 128);
+            if (once)
+                bulk_g2s_hint(d, src + h * kBlockTokens * 128, valid[j] * 128, bar, l2_evict_first());
+            else
+                bulk_g2s(d, src + h * kBlockTokens * 128, valid[j] * 128, bar);
+        }
     }
 }
 
@@ -1547,6 +1551,10 @@ __device__ void tc_stream(const DecodeArgs& a, CtlTc& c, uint8_t* ring) {
         if (*reinterpret_cast<volatile int*>(&c.unit[q]) < 0) return;
         const int n_tiles = *reinterpret_cast<volatile int*>(&c.desc[q][U_N_TILES]);
         const int kvh = *reinterpret_cast<volatile int*>(&c.desc[q][U_KVH]);
+        // the unit's rows are its item's only row block (fewer than a full
+        // tile from row 0): no other unit reads this chunk
+        const bool once = a.kv_read_once && *reinterpret_cast<volatile int*>(&c.desc[q][U_ROW0]) == 0 &&
+                          *reinterpret_cast<volatile int*>(&c.desc[q][U_N_ROWS]) < kTcRows;
         const volatile int* tw = c.tiles[q];
         const int n_pairs = (n_tiles + 1) / 2;
         int kj = 0, vj = 0;
@@ -1557,7 +1565,7 @@ __device__ void tc_stream(const DecodeArgs& a, CtlTc& c, uint8_t* ring) {
             if (kj < n_pairs && mbar_test(smem_u32(&c.s_full[ks]), kph ^ 1)) {  // K slot read by Q.K^T
                 const int32_t w[2] = {tw[2 * kj], 2 * kj + 1 < n_tiles ? tw[2 * kj + 1] : -1};
                 fence_proxy_async();
-                issue_half<HD>(a, kvh, 0, ring + ks * TcSmem<HD>::kStageBytes, w, smem_u32(&c.kfull[ks]));
+                issue_half<HD>(a, kvh, 0, ring + ks * TcSmem<HD>::kStageBytes, w, smem_u32(&c.kfull[ks]), once);
                 if (++ks == kStages) {
                     ks = 0;
                     kph ^= 1;
@@ -1569,7 +1577,7 @@ __device__ void tc_stream(const DecodeArgs& a, CtlTc& c, uint8_t* ring) {
                 const int32_t w[2] = {tw[2 * vj], 2 * vj + 1 < n_tiles ? tw[2 * vj + 1] : -1};
                 fence_proxy_async();
                 issue_half<HD>(a, kvh, 1, ring + vs * TcSmem<HD>::kStageBytes + (HD / 64) * kStageTokens * 128, w,
-                               smem_u32(&c.vfull[vs]));
+                               smem_u32(&c.vfull[vs]), once);
                 if (++vs == kStages) {
                     vs = 0;
                     vph ^= 1;
