@@ -32,7 +32,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "tree-decode leaf-queries/s; HBM GB/s on unique KV bytes vs GB300 peak"
 UNIT = "leaf-queries/s"
-DEFAULT_WORKLOAD = "qwen7b"
+DEFAULT_WORKLOAD = "random_divergence"
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
