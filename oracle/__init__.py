@@ -12,6 +12,8 @@ Contents
                      materialised path (``attention.c``; definition in its
                      header). TreePO's trajectory is s_1 (+) ... (+) s_j
                      (Sec. 2.3) and a decode step attends to all of it.
+``path_scores``      the fp64 scores q.k / sqrt(d) that softmax runs over
+                     (for tests that locate a path's score maximum).
 ``lse_merge``        fp64 log-sum-exp merge of attention partials over
                      disjoint token sets (a split of the path).
 ``OracleForest``     plain tree model: replays a workload script (root,
@@ -96,6 +98,28 @@ def path_attention(q, k, v) -> Tuple[np.ndarray, np.ndarray]:
     if rc != 0:
         raise ValueError(f"oracle_path_attention rejected its arguments (N={n}, Hq={hq}, Hkv={hkv}, d={d})")
     return out, lse
+
+
+def path_scores(q, k) -> np.ndarray:
+    """fp64 attention scores of one decode query over one materialised path.
+
+    q: [Hq][d] bf16; k: [N][Hkv][d] bf16 (root first). Returns s [Hq][N] with
+    s[h][j] = (q_h . k_{j, h // g}) / sqrt(d), g = Hq / Hkv: the scores whose
+    softmax ``path_attention`` takes (step 4 of the definition in
+    ``attention.c``), so LSE = ln sum_j exp(s[h][j]). The tests read them to
+    show where a path's score maximum lies.
+    """
+    qb, kb = bf16_bits(q), bf16_bits(k)
+    q64 = (qb.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    k64 = (kb.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    hq, d = q64.shape
+    n, hkv, d2 = k64.shape
+    assert d2 == d and hq % hkv == 0
+    g = hq // hkv
+    s = np.empty((hq, n), dtype=np.float64)
+    for h in range(hq):
+        s[h] = k64[:, h // g, :] @ q64[h]
+    return s / np.sqrt(d)
 
 
 def lse_merge(parts: Sequence[Tuple[np.ndarray, np.ndarray]]) -> Tuple[np.ndarray, np.ndarray]:

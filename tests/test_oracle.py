@@ -129,6 +129,48 @@ def test_large_scores_do_not_overflow(order):
     np.testing.assert_allclose(o[0], expect, atol=1e-15)
 
 
+def test_path_scores_hand_examples():
+    # two-token golden: q = (2,0,0,0), d = 4, k_1 = 0, k_2 = e_1 -> s = (0, 1)
+    g = golden("two_token.json")
+    s = oracle.path_scores(bf16(g["q"]), bf16(g["k"]))
+    np.testing.assert_array_equal(s, [[0.0, 1.0]])
+    # q = (1,2,0,...), k = (3,-1,0,...), d = 16 -> s = (3 - 2) / 4
+    q = torch.zeros(1, 16)
+    q[0, 0], q[0, 1] = 1, 2
+    k = torch.zeros(1, 1, 16)
+    k[0, 0, 0], k[0, 0, 1] = 3, -1
+    assert oracle.path_scores(q.to(torch.bfloat16), k.to(torch.bfloat16))[0, 0] == 0.25
+
+
+@pytest.mark.parametrize("hq,hkv,d,n", [(4, 1, 64, 37), (28, 4, 128, 129), (6, 3, 32, 2)])
+def test_path_scores_match_torch_and_give_the_oracle_lse(hq, hkv, d, n):
+    # torch's fp64 product over the GQA-expanded path, and the C oracle's LSE
+    # as the log-sum-exp of the scores (two independent routes)
+    gen = torch.Generator().manual_seed(hq + 7 * n)
+    q = rand_bf16(gen, hq, d)
+    k = rand_bf16(gen, n, hkv, d) * 3
+    v = rand_bf16(gen, n, hkv, d)
+    s = oracle.path_scores(q, k)
+    kk = k.double().permute(1, 0, 2).repeat_interleave(hq // hkv, dim=0)      # [Hq][N][d]
+    ref = torch.einsum("hd,hnd->hn", q.double(), kk) / math.sqrt(d)
+    np.testing.assert_allclose(s, ref.numpy(), rtol=0, atol=1e-12)
+    _, lse = oracle.path_attention(q, k, v)
+    np.testing.assert_allclose(torch.logsumexp(torch.from_numpy(s), dim=-1).numpy(), lse, rtol=0, atol=1e-12)
+
+
+def test_path_scores_use_contiguous_gqa_groups():
+    # kv head c holds k = (c+1) e_0, q = e_0: q-head h scores (h // g + 1) / sqrt(d)
+    hq, hkv, d = 6, 3, 16
+    q = torch.zeros(hq, d)
+    q[:, 0] = 1
+    k = torch.zeros(2, hkv, d)
+    for c in range(hkv):
+        k[:, c, 0] = c + 1
+    s = oracle.path_scores(q.to(torch.bfloat16), k.to(torch.bfloat16))
+    for h in range(hq):
+        np.testing.assert_array_equal(s[h], (h // 2 + 1) / 4.0)
+
+
 @pytest.mark.parametrize("cuts", [[1], [5, 64], [31, 32, 33, 200], list(range(1, 299, 7))])
 def test_lse_merge_of_any_split_equals_whole(cuts):
     gen = torch.Generator().manual_seed(len(cuts))
