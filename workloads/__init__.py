@@ -34,7 +34,7 @@ import numpy as np
 import torch
 
 __all__ = [
-    "Heads", "Script", "tiny", "qwen7b", "random_divergence", "wide_prefix",
+    "Heads", "Script", "Peaks", "peaked", "root_appends", "last_appends", "tiny", "qwen7b", "random_divergence", "wide_prefix",
     "no_sharing", "random_tree", "single_path", "shared_prompt", "by_name", "CONFIG_NAMES",
 ]
 
@@ -70,25 +70,32 @@ class Script:
     leaves: List[int]                 # script node ids decoded, in output order
     kv_len: List[int]                 # tokens carried by each kv_id
     description: str = ""
+    shape: Optional["Peaks"] = None   # peaked-score shaping of the draws (None: plain N(0,1))
 
     # ---- tensors -------------------------------------------------------
     def kv(self, kv_id: int, device="cpu") -> Tuple[torch.Tensor, torch.Tensor]:
-        """K, V of append ``kv_id``: bf16 [n][Hkv][hd], i.i.d. N(0,1)."""
+        """K, V of append ``kv_id``: bf16 [n][Hkv][hd], i.i.d. N(0,1) (K
+        reshaped by ``shape`` when set)."""
         n = self.kv_len[kv_id]
         h = self.heads
         g = torch.Generator(device=device)
         g.manual_seed(_mix(self.seed, 1, kv_id))
         k = torch.randn((n, h.num_kv_heads, h.head_dim), generator=g, device=device, dtype=torch.float32)
         v = torch.randn((n, h.num_kv_heads, h.head_dim), generator=g, device=device, dtype=torch.float32)
+        if self.shape is not None:
+            k = self.shape.shape_k(k, kv_id)
         return k.to(torch.bfloat16), v.to(torch.bfloat16)
 
     def q(self, device="cpu", n: Optional[int] = None) -> torch.Tensor:
-        """Decode queries: bf16 [len(leaves)][Hq][hd], i.i.d. N(0,1)."""
+        """Decode queries: bf16 [len(leaves)][Hq][hd], i.i.d. N(0,1) (reshaped
+        by ``shape`` when set)."""
         n = len(self.leaves) if n is None else n
         h = self.heads
         g = torch.Generator(device=device)
         g.manual_seed(_mix(self.seed, 2, 0))
         q = torch.randn((n, h.num_q_heads, h.head_dim), generator=g, device=device, dtype=torch.float32)
+        if self.shape is not None:
+            q = self.shape.shape_q(q)
         return q.to(torch.bfloat16)
 
     # ---- structure summaries (no attention arithmetic) ------------------
@@ -136,6 +143,65 @@ class Script:
 
     def total_appended_tokens(self) -> int:
         return int(sum(self.kv_len))
+
+
+@dataclasses.dataclass(frozen=True)
+class Peaks:
+    """Peaked attention scores, as trained models produce them, from the same
+    seeded draws: every element is transformed before the bf16 rounding.
+
+      Q <- q_scale * Q + q_shift
+      K <- k_scale * K + (ramp * t / (n - 1) + spike * [t in spikes]) * 1
+
+    with 1 the all-ones vector, t the token index inside its append of n
+    tokens. With q_shift > 0 every query has a component along 1, so a ramp
+    makes the scores climb along the append (its maximum keeps moving to
+    later tokens) and a spike makes one token dominate its path. ``ramp_ids``
+    limits the ramp to those appends (None: every append); ``spikes`` maps an
+    append to the token indices that carry the spike.
+    """
+
+    q_scale: float = 1.0
+    k_scale: float = 1.0
+    q_shift: float = 0.0
+    ramp: float = 0.0
+    ramp_ids: Optional[frozenset] = None
+    spike: float = 0.0
+    spikes: Tuple[Tuple[int, Tuple[int, ...]], ...] = ()
+
+    def shape_q(self, q: torch.Tensor) -> torch.Tensor:
+        return q * self.q_scale + self.q_shift
+
+    def shape_k(self, k: torch.Tensor, kv_id: int) -> torch.Tensor:
+        k = k * self.k_scale
+        n = k.shape[0]
+        add = torch.zeros(n, device=k.device, dtype=torch.float32)
+        if self.ramp and (self.ramp_ids is None or kv_id in self.ramp_ids):
+            add += self.ramp * torch.arange(n, device=k.device, dtype=torch.float32) / max(n - 1, 1)
+        for kid, toks in self.spikes:
+            if kid == kv_id:
+                add[list(toks)] += self.spike
+        return k + add[:, None, None]
+
+
+def peaked(script: Script, shape: Peaks) -> Script:
+    """The same workload (same tree, same seeds) with its draws reshaped."""
+    return dataclasses.replace(script, shape=shape, name=script.name + "_peaked")
+
+
+def root_appends(script: Script) -> frozenset:
+    """kv_ids appended to root nodes (the prompts, the longest shared prefixes)."""
+    roots = {op[1] for op in script.ops if op[0] == "root"}
+    return frozenset(op[2] for op in script.ops if op[0] == "append" and op[1] in roots)
+
+
+def last_appends(script: Script) -> dict:
+    """Decoded leaf -> kv_id of the last append on it (the deepest tokens of its path)."""
+    last = {}
+    for op in script.ops:
+        if op[0] == "append":
+            last[op[1]] = op[2]
+    return {lf: last[lf] for lf in script.leaves if lf in last}
 
 
 # --------------------------------------------------------------------------
