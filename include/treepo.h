@@ -87,16 +87,26 @@ typedef struct {
 } tp_config;
 
 /* Bytes the pool arena must hold: pool_blocks * 2 * num_kv_heads *
- * block_tokens * head_dim * 2 (bf16 K and V). Returns -1 on a bad config. */
+ * block_tokens * head_dim * 2 (bf16 K and V). The pool is the KV cache of
+ * every segment of the forest, each stored once (Sec. 2.1). Returns -1 on a
+ * bad config. */
 int64_t tp_pool_bytes(const tp_config* cfg);
 
-/* Create an empty forest over cfg's pool. *out receives the handle. */
+/* Create an empty forest over cfg's pool: the batch of prompt trees one
+ * rollout grows (Sec. 2.2, Algorithm 1 samples every query of a batch as a
+ * tree; Sec. 2.1, their shared prefixes live once in one paged pool).
+ * *out receives the handle. Errors: TP_ERR_INVALID_ARG (bad config),
+ * TP_ERR_OOM / TP_ERR_CUDA (library scratch). */
 tp_status tp_tree_create(const tp_config* cfg, tp_tree** out);
 
-/* Destroy the forest; waits for its device work first. NULL is a no-op. */
+/* Destroy the forest at the end of a rollout (Sec. 2.2: the batch's trees
+ * are done once every path has stopped); waits for its device work first
+ * and frees the library's scratch, not the caller's pool arena. NULL is a
+ * no-op. */
 tp_status tp_tree_destroy(tp_tree* tree);
 
-/* Use another stream for subsequent device work (cudaStream_t; NULL = default). */
+/* Use another stream for subsequent device work (cudaStream_t; NULL =
+ * default). Plumbing with no counterpart in the paper. */
 tp_status tp_set_stream(tp_tree* tree, void* cuda_stream);
 
 /* New tree: an empty root node (a prompt at depth 0, Sec. 2.2). */
@@ -133,10 +143,15 @@ tp_status tp_fork(tp_tree* tree, tp_node node, int32_t k, tp_node* out_children)
 tp_status tp_prune(tp_tree* tree, tp_node leaf);
 
 /*
- * Decode attention for n leaf queries. Row i of Q (device bf16
- * [n][num_q_heads][head_dim]) attends over every token on the root-to-leaf
- * path of leaves[i] (host array; a leaf may appear more than once, each
- * occurrence is its own row). Per q-head h (kv head c):
+ * Decode attention for n leaf queries: the next-token step of every live
+ * path in one segment-level inference step (Sec. 2.2, Algorithm 1). Row i
+ * of Q (device bf16 [n][num_q_heads][head_dim]) attends over every token on
+ * the root-to-leaf path of leaves[i] -- its trajectory so far, the
+ * concatenation s_1 (+) ... (+) s_j of the path's segments (Sec. 2.3) -- and
+ * every prefix segment shared by several listed leaves is read once for all
+ * of them (Sec. 2.1 and Sec. 1: shared prefixes computed once). leaves is a
+ * host array; a leaf may appear more than once, each occurrence is its own
+ * row. Per q-head h (kv head c):
  *   s_j = q_h . k_{j,c} / sqrt(head_dim),  LSE = ln sum_j exp(s_j),
  *   O   = sum_j exp(s_j - LSE) v_{j,c}.
  * O: device bf16 [n][num_q_heads][head_dim]; LSE: device fp32
@@ -182,14 +197,15 @@ tp_status tp_decode_ex(tp_tree* tree, const tp_node* leaves, int32_t n, const vo
  *   - A call whose schedule plus fp32 partials need more than
  *     TP_NOALLOC_SCRATCH_BYTES returns TP_ERR_OOM and launches nothing.
  *   - The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress, with that device current); make that first
- *     call before any stream capture.
+ *     (cudaGetSymbolAddress, with that device current).
  *   - Every call in the process shares the one array and it keeps the last
  *     call's contents; the unit counters that must start at zero are
  *     cleared by each call. Calls whose device work overlaps -- on two
  *     streams, or from two trees -- race on the array and must not overlap.
- *   - The schedule is copied from pageable host memory, so the call waits
- *     for the tree's stream to drain that far before it returns.
+ *   - The schedule is copied from a host buffer that lives only for the
+ *     call (pageable memory, staged by the driver before the call returns),
+ *     so the call is refused with TP_ERR_INVALID_ARG, launching nothing,
+ *     while the tree's stream is being captured into a CUDA graph.
  */
 #define TP_NOALLOC_SCRATCH_BYTES (32ll << 20)
 tp_status tp_decode_noalloc(tp_tree* tree, const tp_node* leaves, int32_t n, const void* Q, void* O,
@@ -273,7 +289,8 @@ tp_status tp_debug_wait_probe(tp_tree* tree, int64_t limit_ns);
 tp_status tp_sync(tp_tree* tree);
 
 /* Message for the last failed call on `tree` (or of tp_tree_create when
- * tree == NULL). Valid until the next call on that tree. */
+ * tree == NULL). Valid until the next call on that tree. Error reporting,
+ * no counterpart in the paper. */
 const char* tp_last_error(tp_tree* tree);
 
 /* Node state. state: 0 live leaf, 1 frozen interior, 2 dead. */
@@ -500,7 +517,8 @@ tp_status tp_tree_advantage(const int32_t* parent, int32_t n_nodes, const int32_
 
 /* ---- inspection (tests and tools) ------------------------------------ */
 
-/* Pool slot of every token on leaf's root-to-leaf path, root first.
+/* Pool slot of every token on leaf's root-to-leaf path (its trajectory
+ * s_1 (+) ... (+) s_j, Sec. 2.3), root first.
  * slots: host int64 [cap]; *n receives the path length (slots untouched
  * beyond cap; TP_ERR_INVALID_ARG if cap < length). */
 tp_status tp_debug_path(tp_tree* tree, tp_node leaf, int64_t* slots, int64_t cap, int64_t* n);
@@ -539,8 +557,9 @@ tp_status tp_debug_schedule(tp_tree* tree, const tp_node* leaves, int32_t n, uin
  * [10] = 1 and two more sections at the end: unit_pos [n_units] (path
  * position of each unit's first token) and vis [n] (tokens of its path that
  * occurrence i -- query token i -- may see). Occurrences are the query
- * tokens; every unit is an mma.sync unit; a unit row whose occurrence sees
- * nothing of the unit is computed but has no merge entry. */
+ * tokens; units are tcgen05 units (mma.sync units with TP_MMA_SYNC); a unit
+ * row whose occurrence sees nothing of the unit is computed but has no merge
+ * entry. */
 tp_status tp_debug_prefill_schedule(tp_tree* tree, const tp_node* nodes, const int32_t* n_queries, int32_t n,
                                     uint32_t flags, int32_t* buf, int64_t cap, int64_t* len);
 

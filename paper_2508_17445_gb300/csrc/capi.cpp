@@ -5,11 +5,23 @@
 #include <new>
 #include <string>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "forest.h"
 
 using tp::fail;
 
 namespace tp {
+
+// One NVTX range per attention call, named for the entry point (a profiler
+// shows each call's host scheduling and launches under it; without a tool
+// attached the push and pop cost a few nanoseconds).
+struct CallRange {
+    explicit CallRange(const char* name) { nvtxRangePushA(name); }
+    ~CallRange() { nvtxRangePop(); }
+    CallRange(const CallRange&) = delete;
+    CallRange& operator=(const CallRange&) = delete;
+};
 
 tp_status cuda_fail(tp_tree* t, cudaError_t e, const char* what) {
     return fail(t, TP_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
@@ -559,6 +571,7 @@ tp_status tp_prune(tp_tree* t, tp_node leaf) {
 
 tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void* Q, void* O, float* LSE,
                        uint32_t flags) {
+    const tp::CallRange range("tp_decode_ex");
     if (!t) return TP_ERR_INVALID_ARG;
     if (n < 0) return fail(t, TP_ERR_INVALID_ARG, "n < 0");
     if (n == 0) return TP_OK;
@@ -598,6 +611,7 @@ tp_status tp_decode_ex(tp_tree* t, const tp_node* leaves, int32_t n, const void*
 
 tp_status tp_prefill(tp_tree* t, const tp_node* nodes, const int32_t* n_queries, int32_t n, const void* Q, void* O,
                      float* LSE, uint32_t flags) {
+    const tp::CallRange range("tp_prefill");
     if (!t) return TP_ERR_INVALID_ARG;
     if (n < 0) return fail(t, TP_ERR_INVALID_ARG, "n < 0");
     if (n == 0) return TP_OK;
@@ -669,6 +683,7 @@ extern "C" {
 
 tp_status tp_decode_host(tp_tree* t, const tp_node* leaves, int32_t n, const void* Q_host, void* O_host,
                          float* LSE_host, uint32_t flags) {
+    const tp::CallRange range("tp_decode_host");
     if (!t) return TP_ERR_INVALID_ARG;
     if (n < 0) return fail(t, TP_ERR_INVALID_ARG, "n < 0");
     if (n == 0) return TP_OK;
@@ -682,6 +697,7 @@ tp_status tp_decode_host(tp_tree* t, const tp_node* leaves, int32_t n, const voi
 
 tp_status tp_prefill_host(tp_tree* t, const tp_node* nodes, const int32_t* n_queries, int32_t n, const void* Q_host,
                           void* O_host, float* LSE_host, uint32_t flags) {
+    const tp::CallRange range("tp_prefill_host");
     if (!t) return TP_ERR_INVALID_ARG;
     if (n < 0) return fail(t, TP_ERR_INVALID_ARG, "n < 0");
     if (n == 0) return TP_OK;
@@ -791,6 +807,7 @@ extern "C" {
 
 tp_status tp_decode_noalloc(tp_tree* t, const tp_node* leaves, int32_t n, const void* Q, void* O, float* LSE,
                             uint32_t flags) {
+    const tp::CallRange range("tp_decode_noalloc");
     if (!t) return TP_ERR_INVALID_ARG;
     if (n < 0) return fail(t, TP_ERR_INVALID_ARG, "n < 0");
     if (n == 0) return TP_OK;
@@ -798,6 +815,13 @@ tp_status tp_decode_noalloc(tp_tree* t, const tp_node* leaves, int32_t n, const 
     if (!t->cfg.pool) return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree cannot decode");
     if (!Q || !O || !LSE || !aligned(Q, 16) || !aligned(O, 16) || !aligned(LSE, 4))
         return fail(t, TP_ERR_INVALID_ARG, "Q/O must be 16-byte and LSE 4-byte aligned device pointers");
+    // The schedule is uploaded from a host vector that dies on return: a
+    // captured copy node would read it again on every replay. Refuse capture.
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    cudaError_t ce = cudaStreamIsCapturing(t->stream, &cap);
+    if (ce != cudaSuccess) return cuda_fail(t, ce, "stream capture query");
+    if (cap != cudaStreamCaptureStatusNone)
+        return fail(t, TP_ERR_INVALID_ARG, "tp_decode_noalloc cannot run while its stream is being captured");
     tp::Schedule S;  // host-side only; the tree's schedule cache is left alone
     tp_status st = tp::build_schedule(t, leaves, n, flags & ~TP_DECODE_NO_CACHE, S);
     if (st != TP_OK) return st;

@@ -70,3 +70,35 @@ def test_noalloc_rejects_work_beyond_its_scratch():
     assert e.value.code == "OOM" and "static scratch" in str(e.value)
     f.sync()
     f.close()
+
+
+def test_noalloc_is_refused_while_its_stream_is_captured():
+    # The schedule goes up from a host buffer that lives only for the call; a
+    # copy captured into a CUDA graph would re-read it on every replay, so the
+    # call refuses a capturing stream, launches nothing, and works again after.
+    script = workloads.qwen7b(seed=6, n_prompts=1)
+    f, leaves = _forest(script)
+    Q = script.q(DEV)
+    O_ref, LSE_ref = f.decode(leaves, Q)
+    O, LSE = torch.empty_like(O_ref), torch.empty_like(LSE_ref)
+    tp.tp_decode_noalloc(f.handle, leaves, Q, O, LSE)  # first call on the device: before any capture
+    f.sync()
+    side = torch.cuda.Stream()
+    tp.tp_set_stream(f.handle, side.cuda_stream)
+    graph = torch.cuda.CUDAGraph()
+    x = torch.zeros(1, device=DEV)
+    with torch.cuda.graph(graph, stream=side):
+        x.add_(1)
+        with pytest.raises(tp.TreepoError) as e:
+            tp.tp_decode_noalloc(f.handle, leaves, Q, O, LSE)
+    assert e.value.code == "INVALID_ARG" and "captured" in str(e.value)
+    graph.replay()
+    torch.cuda.synchronize()
+    assert x.item() == 1.0                              # the graph holds only the torch op
+    tp.tp_set_stream(f.handle, torch.cuda.current_stream().cuda_stream)
+    O.fill_(float("nan"))
+    tp.tp_decode_noalloc(f.handle, leaves, Q, O, LSE)
+    f.sync()
+    assert (O.float() - O_ref.float()).abs().max().item() <= TOL_O
+    assert (LSE - LSE_ref).abs().max().item() <= TOL_LSE
+    f.close()
