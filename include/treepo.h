@@ -32,6 +32,14 @@
  * bounded wait that runs out sets a device flag that tp_sync() reports as
  * TP_ERR_DEVICE.
  *
+ * Bounds-checked build. libtreepo_checked.so (build.py builds it beside
+ * libtreepo.so, compiled with TP_BOUNDS_CHECK) exports the same calls; its
+ * kernels check every index they take from a schedule or a slot list
+ * before the access (see tp_debug_check_schedule) and, on a failed check,
+ * skip the access and set a device flag that tp_sync() reports as
+ * TP_ERR_DEVICE. It is a debugging aid: on valid input it computes the same
+ * results as libtreepo.so, a little slower.
+ *
  * Pointer conventions. "device" = CUDA device memory (any allocator); "host"
  * = ordinary host memory. The caller owns every buffer it passes; the library
  * keeps no pointer to a caller buffer after a call returns, except the pool
@@ -56,7 +64,8 @@ typedef int32_t tp_status;
 #define TP_ERR_NOT_LEAF (-5)    /* decode/prune of an interior node                */
 #define TP_ERR_EMPTY_PATH (-6)  /* decode of a leaf whose path holds no token      */
 #define TP_ERR_CUDA (-7)        /* a CUDA runtime call failed                      */
-#define TP_ERR_DEVICE (-8)      /* a kernel's bounded wait ran out (tp_sync)       */
+#define TP_ERR_DEVICE (-8)      /* a kernel's bounded wait ran out, or (bounds-    */
+                                /* checked build) an index failed its check        */
 
 typedef int32_t tp_node;
 typedef struct tp_tree tp_tree;
@@ -552,6 +561,23 @@ tp_status tp_debug_gather(tp_tree* tree, tp_node leaf, void* K_out, void* V_out,
  */
 tp_status tp_debug_schedule(tp_tree* tree, const tp_node* leaves, int32_t n, uint32_t flags,
                             int32_t* buf, int64_t cap, int64_t* len);
+
+/*
+ * Check a schedule (the word layout of tp_debug_schedule and
+ * tp_debug_prefill_schedule) on the host with the index predicates that the
+ * bounds-checked build of the kernels applies before every access: each
+ * unit record's tiles inside the tile section (at most 128), its kind in
+ * launch order, its rows' occurrence entries inside the occurrence list and
+ * their partial slots below n_slots (slot_base -1 only in prefill
+ * schedules), its kv head below num_kv_heads; each tile word's block below
+ * the tree's pool_blocks with 1..32 valid tokens; each occurrence entry
+ * below n; each occurrence's merge range inside the merge list; each merge
+ * slot below n_slots. violations: host int64 [5] receives the number of bad
+ * unit records, tile words, occurrence entries, merge ranges and merge
+ * slots. Errors: TP_ERR_INVALID_ARG (not a schedule: bad magic, bad header,
+ * shorter than its header says).
+ */
+tp_status tp_debug_check_schedule(tp_tree* tree, const int32_t* words, int64_t n_words, int64_t* violations);
 
 /* The schedule tp_prefill would run, in the layout above with header word
  * [10] = 1 and two more sections at the end: unit_pos [n_units] (path

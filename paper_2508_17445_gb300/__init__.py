@@ -23,7 +23,7 @@ __all__ = [
     "tp_set_stream", "tp_add_root", "tp_append_segment", "tp_fork", "tp_prune", "tp_decode", "tp_decode_ex",
     "tp_sync", "tp_last_error", "tp_get_node_info", "tp_get_stats", "tp_profile_start", "tp_profile_stop",
     "tp_debug_path", "tp_debug_gather",
-    "tp_debug_schedule", "tp_decode_noalloc", "tp_append_tokens", "tp_synth_tokens", "tp_branch_assign",
+    "tp_debug_schedule", "tp_debug_check_schedule", "tp_decode_noalloc", "tp_append_tokens", "tp_synth_tokens", "tp_branch_assign",
     "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "tp_prefill", "tp_debug_prefill_schedule", "tp_decode_host", "tp_prefill_host", "tp_debug_wait_probe", "TpRolloutParams", "TpRolloutStats",
     "TpRolloutProbe", "rollout_params", "TP_BRANCH_EVEN", "TP_BRANCH_LOGP_HIGH", "TP_BRANCH_LOGP_LOW",
     "EVENT_NAMES", "TP_SEG_EOS", "TP_SEG_BOXED", "TP_SEG_FAILED", "TP_SEG_MAX_DEPTH", "Forest", "TP_DECODE_NO_SHARE", "TP_DECODE_CUDA_CORE_SMALL", "TP_DECODE_NO_CACHE", "TP_DECODE_TCGEN05", "TP_DECODE_ALL_TCGEN05", "TP_MMA_SYNC",
@@ -31,7 +31,10 @@ __all__ = [
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_LIB_PATH = os.path.join(_HERE, "libtreepo.so")
+# TREEPO_BOUNDS_CHECK=1 selects the bounds-checked build (same ABI; every
+# kernel checks its schedule indices before each access)
+BOUNDS_CHECKED = os.environ.get("TREEPO_BOUNDS_CHECK", "0") == "1"
+_LIB_PATH = os.path.join(_HERE, "libtreepo_checked.so" if BOUNDS_CHECKED else "libtreepo.so")
 _lib: Optional[ctypes.CDLL] = None
 
 TP_DECODE_NO_SHARE = 1
@@ -57,6 +60,7 @@ EXPORTED_SYMBOLS = (
     "tp_debug_gather", "tp_debug_schedule", "tp_decode_noalloc", "tp_append_tokens", "tp_synth_tokens",
     "tp_branch_assign", "tp_rollout", "tp_advantage_workspace_bytes", "tp_tree_advantage", "tp_prefill",
     "tp_debug_prefill_schedule", "tp_decode_host", "tp_prefill_host", "tp_debug_wait_probe",
+    "tp_debug_check_schedule",
 )
 
 
@@ -121,7 +125,8 @@ def load_library() -> ctypes.CDLL:
     if _lib is not None:
         return _lib
     if not os.path.exists(_LIB_PATH):
-        raise ImportError(f"{_LIB_PATH} is missing: run `python -m paper_2508_17445_gb300.build` "
+        flag = " --checked" if BOUNDS_CHECKED else ""
+        raise ImportError(f"{_LIB_PATH} is missing: run `python -m paper_2508_17445_gb300.build{flag}` "
                           "(there is no fallback implementation)")
     lib = ctypes.CDLL(_LIB_PATH)
     P, I32, I64, U32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32
@@ -157,6 +162,7 @@ def load_library() -> ctypes.CDLL:
         "tp_prefill_host": (I32, [P, P, P, I32, P, P, P, U32]),
         "tp_debug_wait_probe": (I32, [P, I64]),
         "tp_debug_prefill_schedule": (I32, [P, P, P, I32, U32, P, I64, P]),
+        "tp_debug_check_schedule": (I32, [P, P, I64, P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -370,6 +376,18 @@ def tp_debug_schedule(h, leaves: Sequence[int], flags: int = 0) -> Dict[str, np.
     _check(h, lib.tp_debug_schedule(h, arr.ctypes.data if len(arr) else None, len(arr), flags,
                                      buf.ctypes.data, len(buf), ctypes.byref(n_words)))
     return _parse_schedule(buf[: n_words.value])
+
+
+CHECK_CATEGORIES = ("units", "tiles", "occ", "merge_ranges", "merge_slots")
+
+
+def tp_debug_check_schedule(h, words: np.ndarray) -> Dict[str, int]:
+    """Violation counts of a schedule's words under the bounds-checked
+    kernels' index predicates (zero everywhere for a valid schedule)."""
+    w = np.ascontiguousarray(np.asarray(words, dtype=np.int32))
+    out = (ctypes.c_int64 * 5)()
+    _check(h, load_library().tp_debug_check_schedule(h, w.ctypes.data, len(w), out))
+    return dict(zip(CHECK_CATEGORIES, (int(x) for x in out)))
 
 
 def tp_append_tokens(h, nodes: Sequence[int], K=None, V=None) -> None:

@@ -173,6 +173,9 @@ tp_status rollout_token_step(tp_tree* t, const tp_node* nodes, int32_t n, int32_
         a.pos = pos;
         a.n = n;
         a.n_pairs = n_pairs;
+        a.err = t->d_err;
+        a.pool_blocks = t->cfg.pool_blocks;
+        a.sched_words = (int64_t)t->sched.words.size();
         LaunchTimer timer(t, KK_APPEND);
         cudaError_t e = launch_rollout_step(t->cfg.head_dim, a, t->stream);
         if (e != cudaSuccess) st = cuda_fail(t, e, "rollout step kernel");
@@ -213,6 +216,20 @@ tp_status ensure_device(tp_tree* t, T*& ptr, int64_t& cap, int64_t need, const c
 
 tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O, float* LSE);
 
+// What a schedule's words index into (checked by the bounds-checked build).
+tp::Extents extents_of(const tp_tree* t, const tp::Schedule& S) {
+    tp::Extents x;
+    x.pool_blocks = t->cfg.pool_blocks;
+    x.n_tiles = S.n_tiles;
+    x.n_occ = S.n_occ;
+    x.n = S.n;
+    x.n_slots = S.n_slots;
+    x.n_merge = S.n_merge;
+    x.hkv = t->cfg.num_kv_heads;
+    x.group = t->cfg.num_q_heads / t->cfg.num_kv_heads;
+    return x;
+}
+
 tp_status upload_schedule(tp_tree* t, const tp::Schedule& s) {
     const int64_t words = (int64_t)s.words.size();
     tp_status st = ensure_device(t, t->d_sched, t->d_sched_cap, words, "schedule buffer");
@@ -229,7 +246,7 @@ tp_status patch_cached_schedule(tp_tree* t) {
     if (st != TP_OK) return st;
     st = stage_upload(t, t->d_patch, t->patch_words.data(), 2 * (int64_t)n);
     if (st != TP_OK) return st;
-    cudaError_t e = tp::launch_patch(t->d_sched, t->d_patch, n, t->stream);
+    cudaError_t e = tp::launch_patch(t->d_sched, t->d_patch, n, t->stream, (int64_t)t->sched.words.size(), t->d_err);
     tp::count_kernels(t, tp::KK_DECODE, 1);
     if (e != cudaSuccess) return cuda_fail(t, e, "schedule patch kernel");
     return TP_OK;
@@ -391,6 +408,8 @@ tp_status tp_append_segment(tp_tree* t, tp_node node, int32_t n_tokens, const vo
         a.head_bytes = bt * hd * 2;
         a.block_bytes = (int64_t)2 * hkv * a.head_bytes;
         a.hkv = hkv;
+        a.err = t->d_err;
+        a.pool_blocks = t->cfg.pool_blocks;
         const int64_t row_bytes = (int64_t)hkv * hd * 2;
         int64_t pos = nd.n_tokens;
         const int64_t end = (int64_t)nd.n_tokens + n_tokens;
@@ -451,6 +470,8 @@ tp_status tp_append_tokens(tp_tree* t, const tp_node* nodes, int32_t n, const vo
             a.block_bytes = (int64_t)2 * t->cfg.num_kv_heads * a.head_bytes;
             a.hkv = t->cfg.num_kv_heads;
             a.n = n;
+            a.err = t->d_err;
+            a.pool_blocks = t->cfg.pool_blocks;
             tp::LaunchTimer timer(t, tp::KK_APPEND);
             cudaError_t e = tp::launch_append_tokens(t->cfg.head_dim, a, t->stream);
             if (e != cudaSuccess) st = cuda_fail(t, e, "token append kernel");
@@ -770,6 +791,7 @@ tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O
     a.group = hq / t->cfg.num_kv_heads;
     a.qk_scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
     a.kv_read_once = S.kv_read_once ? 1 : 0;
+    a.ext = extents_of(t, S);
     cudaError_t e = cudaSuccess;
     if (S.n_tc > 0 && S.n_units > S.n_tc && !t->side) {  // concurrent tcgen05 units need a second stream
         e = cudaStreamCreateWithFlags(&t->side, cudaStreamNonBlocking);
@@ -792,6 +814,9 @@ tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O
     m.out = (uint16_t*)O;
     m.lse = LSE;
     m.counters = t->d_err + 1;
+    m.err = t->d_err;
+    m.n_merge = S.n_merge;
+    m.n_slots = S.n_slots;
     m.n = S.n_merge > 0 ? S.n : 0;  // 0: every row was written by its only unit; only re-arm the counters
     m.hq = hq;
     {
@@ -865,6 +890,7 @@ tp_status tp_decode_noalloc(tp_tree* t, const tp_node* leaves, int32_t n, const 
     a.group = hq / t->cfg.num_kv_heads;
     a.qk_scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)hd));
     a.kv_read_once = S.kv_read_once ? 1 : 0;
+    a.ext = extents_of(t, S);
     e = tp::launch_decode(hd, a, t->stream);
     if (e != cudaSuccess) return cuda_fail(t, e, "decode kernel");
     tp::MergeArgs m;
@@ -875,6 +901,9 @@ tp_status tp_decode_noalloc(tp_tree* t, const tp_node* leaves, int32_t n, const 
     m.out = (uint16_t*)O;
     m.lse = LSE;
     m.counters = t->d_err + 1;
+    m.err = t->d_err;
+    m.n_merge = S.n_merge;
+    m.n_slots = S.n_slots;
     m.n = n;
     m.hq = hq;
     e = tp::launch_merge(hd, m, t->stream);
@@ -942,7 +971,10 @@ tp_status tp_sync(tp_tree* t) {
     if (e != cudaSuccess) return cuda_fail(t, e, "error flag read");
     if (flag) {
         cudaMemset(t->d_err, 0, sizeof(int32_t));
-        return fail(t, TP_ERR_DEVICE, "a kernel gave up a bounded wait (flag " + std::to_string(flag) + ")");
+        std::string what;
+        if (flag & tp::kErrBounds) what = "an index failed its bounds check (the access was skipped)";
+        if (flag & ~tp::kErrBounds) what += std::string(what.empty() ? "" : "; ") + "a kernel gave up a bounded wait";
+        return fail(t, TP_ERR_DEVICE, what + " (flag " + std::to_string(flag) + ")");
     }
     return TP_OK;
 }
@@ -1018,6 +1050,8 @@ tp_status tp_debug_gather(tp_tree* t, tp_node leaf, void* K_out, void* V_out, in
     a.hkv = t->cfg.num_kv_heads;
     a.n_tiles = (int32_t)tiles.size();
     a.block_tokens = t->cfg.block_tokens;
+    a.err = t->d_err;
+    a.pool_blocks = t->cfg.pool_blocks;
     {
         tp::LaunchTimer timer(t, tp::KK_GATHER);
         e = tp::launch_gather(t->cfg.head_dim, a, len, t->stream);
@@ -1025,6 +1059,46 @@ tp_status tp_debug_gather(tp_tree* t, tp_node leaf, void* K_out, void* V_out, in
     if (e != cudaSuccess) return cuda_fail(t, e, "gather kernel");
     e = cudaStreamSynchronize(t->stream);  // the host tile list must outlive the copy
     if (e != cudaSuccess) return cuda_fail(t, e, "gather sync");
+    return TP_OK;
+}
+
+tp_status tp_debug_check_schedule(tp_tree* t, const int32_t* w, int64_t n_words, int64_t* violations) {
+    if (!t || !violations) return TP_ERR_INVALID_ARG;
+    if (!w || n_words < tp::kSchedHeaderWords || w[0] != tp::kSchedMagic)
+        return fail(t, TP_ERR_INVALID_ARG, "not a schedule (short buffer or bad magic)");
+    const int32_t n_units = w[1], n_tiles = w[2], n_occ = w[3], n = w[4], n_slots = w[5], n_merge = w[6];
+    const int32_t n_tensor = w[8], n_tc = w[9];
+    const bool prefill = w[10] == 1;
+    if (n_units < 0 || n_tiles < 0 || n_occ < 0 || n < 0 || n_slots < 0 || n_merge < 0 || n_tensor < 0 || n_tc < 0 ||
+        (int64_t)n_tc + n_tensor > n_units)
+        return fail(t, TP_ERR_INVALID_ARG, "bad schedule header");
+    const int64_t off_units = tp::kSchedHeaderWords, off_tiles = off_units + (int64_t)n_units * tp::kUnitWords;
+    const int64_t off_occ = off_tiles + n_tiles, off_moff = off_occ + n_occ, off_mslot = off_moff + n + 1;
+    const int64_t end = off_mslot + n_merge + (prefill ? (int64_t)n_units + n : 0);
+    if (n_words < end) return fail(t, TP_ERR_INVALID_ARG, "schedule shorter than its header says");
+    tp::Extents x;
+    x.pool_blocks = t->cfg.pool_blocks;
+    x.n_tiles = n_tiles;
+    x.n_occ = n_occ;
+    x.n = n;
+    x.n_slots = n_slots;
+    x.n_merge = n_merge;
+    x.hkv = t->cfg.num_kv_heads;
+    x.group = t->cfg.num_q_heads / t->cfg.num_kv_heads;
+    int64_t bad[5] = {0, 0, 0, 0, 0};  // units, tile words, occurrence entries, merge ranges, merge slots
+    for (int32_t k = 0; k < n_units; ++k) {
+        const int32_t* u = w + off_units + (int64_t)k * tp::kUnitWords;
+        // launch order: tcgen05 units, then mma.sync, then CUDA-core units
+        const int32_t kind = k < n_tc ? tp::KIND_TC : k < n_tc + n_tensor ? tp::KIND_TENSOR : tp::KIND_CUDA_CORE;
+        bad[0] += !(u[tp::U_KIND] == kind &&
+                    tp::unit_ok(u[tp::U_TILE_OFF], u[tp::U_N_TILES], u[tp::U_OCC_OFF], u[tp::U_ROW0], u[tp::U_N_ROWS],
+                                u[tp::U_SLOT_BASE], u[tp::U_KVH], tp::unit_rows_limit(kind), prefill, x));
+    }
+    for (int64_t k = 0; k < n_tiles; ++k) bad[1] += !tp::tile_word_ok(w[off_tiles + k], x.pool_blocks);
+    for (int64_t k = 0; k < n_occ; ++k) bad[2] += !tp::in_range(w[off_occ + k], n);
+    for (int32_t i = 0; i < n; ++i) bad[3] += !tp::merge_range_ok(w[off_moff + i], w[off_moff + i + 1], n_merge);
+    for (int64_t k = 0; k < n_merge; ++k) bad[4] += !tp::in_range(w[off_mslot + k], n_slots);
+    std::memcpy(violations, bad, sizeof bad);
     return TP_OK;
 }
 

@@ -44,6 +44,73 @@ constexpr int kMaxUnitTiles = 128;
 constexpr int kCudaCoreMaxRows = 16;
 // Pool blocks an append kernel launch can address (larger appends loop).
 constexpr int kAppendMaxBlocks = 256;
+// Tokens per pool block (the ABI fixes block_tokens to 32).
+constexpr int kTileTokens = 32;
+
+// ---- index checks of the bounds-checked build -----------------------------
+// Built with -DTP_BOUNDS_CHECK (build.py's checked variant), every kernel
+// checks each schedule-derived index before it uses it -- tile words against
+// the pool, unit records against the schedule's sections, occurrence entries
+// against the rows of Q/O, partial slots, merge ranges, pool slots of token
+// appends, schedule patch positions -- and on a failed check sets
+// kErrBounds in the device error word and skips the access (no trap). The
+// predicates are shared with the host, where tp_debug_check_schedule runs
+// them over a schedule without a GPU. In the default build the checks
+// compile away.
+#if defined(__CUDACC__)
+#define TP_HD __host__ __device__ __forceinline__
+#else
+#define TP_HD inline
+#endif
+#ifdef TP_BOUNDS_CHECK
+constexpr bool kBoundsCheck = true;
+#else
+constexpr bool kBoundsCheck = false;
+#endif
+constexpr int32_t kErrBounds = 64;
+
+// Sizes of everything a schedule's words index into.
+struct Extents {
+    int64_t pool_blocks = 0;  // pool blocks
+    int32_t n_tiles = 0;      // tile words
+    int32_t n_occ = 0;        // occurrence-list entries
+    int32_t n = 0;            // leaf occurrences (query rows of Q, O, LSE)
+    int32_t n_slots = 0;      // partial slots
+    int32_t n_merge = 0;      // merge entries
+    int32_t hkv = 0;
+    int32_t group = 1;
+};
+
+TP_HD bool in_range(int64_t i, int64_t n) { return i >= 0 && i < n; }
+
+// Tile word block << 7 | (valid - 1): a pool block and 1..32 valid tokens.
+TP_HD bool tile_word_ok(int32_t w, int64_t pool_blocks) {
+    return w >= 0 && (int64_t)(w >> kTileValidBits) < pool_blocks && (w & ((1 << kTileValidBits) - 1)) < kTileTokens;
+}
+
+// Most query rows a unit of each kind holds.
+TP_HD int32_t unit_rows_limit(int32_t kind) {
+    return kind == KIND_CUDA_CORE ? kCudaCoreMaxRows : kind == KIND_TC ? kTcRowsPerUnit : kTensorRowsPerUnit;
+}
+
+// A unit record: its tiles lie inside the tile section (at most
+// kMaxUnitTiles), its rows' occurrence entries inside the occurrence list,
+// their partial slots below n_slots (slot_base -1: the rows' only unit writes
+// O and LSE directly, prefill schedules only), its kv head below hkv.
+TP_HD bool unit_ok(int32_t tile_off, int32_t n_tiles, int32_t occ_off, int32_t row0, int32_t n_rows,
+                   int32_t slot_base, int32_t kvh, int32_t rows_limit, bool direct_ok, const Extents& x) {
+    if (n_tiles < 1 || n_tiles > kMaxUnitTiles || tile_off < 0 || (int64_t)tile_off + n_tiles > x.n_tiles)
+        return false;
+    if (n_rows < 1 || n_rows > rows_limit || row0 < 0 || occ_off < 0 || kvh < 0 || kvh >= x.hkv || x.group < 1)
+        return false;
+    const int64_t last = ((int64_t)row0 + n_rows - 1) / x.group;  // the unit's last occurrence group
+    if ((int64_t)occ_off + last >= x.n_occ) return false;
+    if (slot_base < 0) return direct_ok && slot_base == -1;
+    return (int64_t)slot_base + last < x.n_slots;
+}
+
+// Occurrence `i`'s merge entries [beg, end).
+TP_HD bool merge_range_ok(int32_t beg, int32_t end, int32_t n_merge) { return 0 <= beg && beg <= end && end <= n_merge; }
 
 // ---- device launch arguments --------------------------------------------
 struct DecodeArgs {
@@ -74,6 +141,7 @@ struct DecodeArgs {
     int32_t kv_read_once = 0;  // decode, default routing: the mma.sync kernel's units, and the tcgen05
                                // units of single-row-block items, read disjoint K/V (copied in as L2
                                // evict-first)
+    Extents ext;  // what the schedule indexes into (bounds-checked build)
 };
 
 struct MergeArgs {
@@ -86,6 +154,9 @@ struct MergeArgs {
     int32_t* counters;  // decode's three unit counters, reset to 0 here
     int32_t n;
     int32_t hq;
+    int32_t* err = nullptr;  // device error word (bounds-checked build)
+    int32_t n_merge = 0;     // merge entries and partial slots (bounds-checked build)
+    int32_t n_slots = 0;
 };
 
 struct AppendArgs {
@@ -97,6 +168,8 @@ struct AppendArgs {
     int32_t hkv;
     int32_t first_row;  // row of the first appended token inside blocks[0]
     int32_t n_tokens;
+    int32_t* err = nullptr;      // bounds-checked build: device error word
+    int64_t pool_blocks = 0;     // and the pool size the blocks are checked against
     int32_t blocks[kAppendMaxBlocks];
 };
 
@@ -110,6 +183,8 @@ struct GatherArgs {
     int32_t hkv;
     int32_t n_tiles;
     int32_t block_tokens;
+    int32_t* err = nullptr;   // bounds-checked build: device error word
+    int64_t pool_blocks = 0;  // and the pool size
 };
 
 // One token per listed node: row i of k / v goes to pool slot slots[i]
@@ -123,6 +198,8 @@ struct AppendTokensArgs {
     int32_t head_bytes;
     int32_t hkv;
     int32_t n;
+    int32_t* err = nullptr;   // bounds-checked build: device error word
+    int64_t pool_blocks = 0;  // and the pool size the slots are checked against
 };
 
 // Synthetic activations of the stand-in model (splitmix.h): row i is token
@@ -154,6 +231,9 @@ struct StepArgs {
     uint64_t seed;
     int64_t block_bytes;
     int32_t head_bytes, hkv, q_width, pos, n, n_pairs;
+    int32_t* err = nullptr;     // bounds-checked build: device error word,
+    int64_t pool_blocks = 0;    // the pool size the slots are checked against
+    int64_t sched_words = 0;    // and the schedule length the patches are
 };
 
 // Tree advantage (Eq. tree_ae) over a node table; see tp_tree_advantage.
@@ -178,8 +258,10 @@ cudaError_t launch_decode(int head_dim, const DecodeArgs& a, cudaStream_t s, cud
                           cudaEvent_t fork = nullptr, cudaEvent_t join = nullptr);
 cudaError_t launch_merge(int head_dim, const MergeArgs& a, cudaStream_t s);
 cudaError_t launch_gather(int head_dim, const GatherArgs& a, int64_t n_tokens, cudaStream_t s);
-// sched[pairs[2k]] = pairs[2k + 1] for k < n.
-cudaError_t launch_patch(int32_t* sched, const int32_t* pairs, int32_t n, cudaStream_t s);
+// sched[pairs[2k]] = pairs[2k + 1] for k < n (sched_words and err: the
+// bounds-checked build's limit and error word).
+cudaError_t launch_patch(int32_t* sched, const int32_t* pairs, int32_t n, cudaStream_t s, int64_t sched_words = 0,
+                         int32_t* err = nullptr);
 cudaError_t launch_wait_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s);
 cudaError_t launch_append_tokens(int head_dim, const AppendTokensArgs& a, cudaStream_t s);
 cudaError_t launch_synth(const SynthArgs& a, cudaStream_t s);

@@ -260,6 +260,17 @@ __device__ __forceinline__ int kv_off(int row, int chunk) {
     return (chunk >> 3) * (ROWS * 128) + row * 128 + (((chunk & 7) ^ (row & 7)) << 4);
 }
 
+// Bounds-checked build: true when an index check passed; otherwise records
+// the failure in the device error word (the caller skips the access). In the
+// default build it is `true` and the check compiles away.
+__device__ __forceinline__ bool check(bool ok, int32_t* err) {
+    if (kBoundsCheck && !ok) {
+        atomicOr(err, kErrBounds);
+        return false;
+    }
+    return true;
+}
+
 // ------------------------------------------------------------------ append --
 template <int HD>
 __global__ void append_kernel(const AppendArgs a) {
@@ -277,6 +288,7 @@ __global__ void append_kernel(const AppendArgs a) {
         const int pos = a.first_row + i;
         const int blk = a.blocks[pos / kBlockTokens];
         const int row = pos % kBlockTokens;
+        if (!check(in_range(blk, a.pool_blocks), a.err)) continue;
         uint8_t* dst = a.pool + (int64_t)blk * a.block_bytes + (int64_t)(kv * a.hkv + h) * a.head_bytes +
                        kv_off<kBlockTokens>(row, c);
         *reinterpret_cast<uint4*>(dst) = val;
@@ -297,6 +309,7 @@ __global__ void append_tokens_kernel(const AppendTokensArgs a) {
         const int h = (int)((r / CH) % a.hkv);
         const int i = (int)(r / ((int64_t)CH * a.hkv));
         const int32_t slot = a.slots[i];
+        if (!check(in_range(slot, a.pool_blocks * kBlockTokens), a.err)) continue;
         const uint4 val = reinterpret_cast<const uint4*>(kv ? a.v : a.k)[r];
         uint8_t* dst = a.pool + (int64_t)(slot / kBlockTokens) * a.block_bytes +
                        (int64_t)(kv * a.hkv + h) * a.head_bytes + kv_off<kBlockTokens>(slot % kBlockTokens, c);
@@ -368,6 +381,7 @@ __global__ void rollout_step_kernel(const StepArgs a) {
             const uint2 x0 = synth_words(splitmix64(a.seed, draw_counter(tag, node, (uint32_t)a.pos, w0)));
             const uint2 x1 = synth_words(splitmix64(a.seed, draw_counter(tag, node, (uint32_t)a.pos, w0 + 1)));
             const int32_t slot = a.slots[i];
+            if (!check(in_range(slot, a.pool_blocks * kBlockTokens), a.err)) continue;
             uint8_t* dst = a.pool + (int64_t)(slot / kBlockTokens) * a.block_bytes +
                            (int64_t)(kv * a.hkv + h) * a.head_bytes + kv_off<kBlockTokens>(slot % kBlockTokens, c);
             *reinterpret_cast<uint4*>(dst) = make_uint4(x0.x, x0.y, x1.x, x1.y);
@@ -379,6 +393,7 @@ __global__ void rollout_step_kernel(const StepArgs a) {
                 synth_words(splitmix64(a.seed, draw_counter(kTagQ, node, (uint32_t)a.pos, (uint32_t)w)));
         } else {
             const int64_t k = idx - kv_items - q_items;
+            if (!check(in_range(a.pairs[2 * k], a.sched_words), a.err)) continue;
             a.sched[a.pairs[2 * k]] = a.pairs[2 * k + 1];
         }
     }
@@ -490,9 +505,9 @@ __global__ void __launch_bounds__(kAdvThreads) advantage_kernel(const AdvantageA
 }
 
 // ------------------------------------------------------- schedule patch --
-__global__ void patch_kernel(int32_t* sched, const int32_t* pairs, int32_t n) {
+__global__ void patch_kernel(int32_t* sched, const int32_t* pairs, int32_t n, int64_t sched_words, int32_t* err) {
     const int k = blockIdx.x * blockDim.x + threadIdx.x;
-    if (k < n) sched[pairs[2 * k]] = pairs[2 * k + 1];
+    if (k < n && check(in_range(pairs[2 * k], sched_words), err)) sched[pairs[2 * k]] = pairs[2 * k + 1];
 }
 
 // ------------------------------------------------------------------ gather --
@@ -519,6 +534,7 @@ __global__ void gather_kernel(const GatherArgs a, int64_t n_tokens) {
         }
         const int row = (int)(tok - base);
         const int64_t blk = w >> kTileValidBits;
+        if (!check(tile_word_ok(w, a.pool_blocks), a.err)) continue;
         const uint8_t* src = a.pool + blk * a.block_bytes + (int64_t)(kv * a.hkv + h) * a.head_bytes +
                              kv_off<kBlockTokens>(row, c);
         reinterpret_cast<uint4*>(kv ? a.v_out : a.k_out)[r] = *reinterpret_cast<const uint4*>(src);
@@ -606,7 +622,7 @@ __device__ __forceinline__ void issue_pair(const DecodeArgs& a, CtlT& c, int kvh
     int valid[2] = {0, 0};
     uint32_t bytes = 0;
     for (int j = 0; j < 2; ++j)
-        if (w[j] >= 0) {
+        if (w[j] >= 0 && check(tile_word_ok(w[j], a.ext.pool_blocks), a.err)) {  // a bad word: a missing tile
             valid[j] = (w[j] & ((1 << kTileValidBits) - 1)) + 1;
             bytes += 2u * (uint32_t)(valid[j] * RB);
         }
@@ -742,7 +758,8 @@ struct CudaCorePath {
             const int rr_ = rg * NR + r;
             if (rr_ < u.n_rows) {
                 const int item_row = u.row0 + rr_;
-                const int occ = a.occ[u.occ_off + item_row / a.group];
+                int occ = a.occ[u.occ_off + item_row / a.group];
+                if (!check(in_range(occ, a.ext.n), a.err)) occ = 0;
                 const int qh = u.kvh * a.group + item_row % a.group;
                 const uint4 w = *reinterpret_cast<const uint4*>(a.q + ((int64_t)occ * a.hq + qh) * HD + dg * 8);
                 const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
@@ -956,7 +973,12 @@ struct TensorPath {
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
                 const int r = mt * 16 + g4 + 8 * h;
-                vis[h] = r < u.n_rows ? a.vis[a.occ[u.occ_off + (u.row0 + r) / a.group]] : 0x7fffffff;
+                if (r >= u.n_rows) {
+                    vis[h] = 0x7fffffff;
+                    continue;
+                }
+                const int occ = a.occ[u.occ_off + (u.row0 + r) / a.group];
+                vis[h] = check(in_range(occ, a.ext.n), a.err) ? a.vis[occ] : 0;
             }
         }
 
@@ -1099,6 +1121,7 @@ struct TensorPath {
             const float inv = 1.f / l_run[h];
             if (CAUSAL && u.slot_base < 0) {  // the row's only unit: final O and LSE
                 const int occ = a.occ[u.occ_off + item_row / a.group];
+                if (!check(in_range(occ, a.ext.n), a.err)) continue;
                 uint16_t* dst = a.out + ((int64_t)occ * a.hq + qh) * HD;
 #pragma unroll
                 for (int j = 0; j < NT; ++j)
@@ -1143,6 +1166,13 @@ __device__ void fetch_units(const DecodeArgs& a, Ctl& c, uint8_t* qbuf) {
         d.slot_base = __shfl_sync(0xffffffffu, word, U_SLOT_BASE);
         d.kvh = __shfl_sync(0xffffffffu, word, U_KVH);
         d.kind = __shfl_sync(0xffffffffu, word, U_KIND);
+        if (kBoundsCheck && u >= 0 &&
+            !(d.kind == (KIND == KIND_CUDA_CORE ? KIND_CUDA_CORE : KIND_TENSOR) &&
+              unit_ok(d.tile_off, d.n_tiles, d.occ_off, d.row0, d.n_rows, d.slot_base, d.kvh,
+                      unit_rows_limit(d.kind), KIND == KIND_PREFILL, a.ext))) {
+            if (lane == 0) atomicOr(a.err, kErrBounds);  // a bad unit record: this CTA takes no more units
+            u = -1;
+        }
         if (u >= 0)
             for (int t = lane; t < d.n_tiles; t += 32) c.tiles[q][t] = a.tiles[d.tile_off + t];
         if (lane == 0) {
@@ -1171,7 +1201,8 @@ __device__ void fetch_units(const DecodeArgs& a, Ctl& c, uint8_t* qbuf) {
             const int g = a.group;
             for (int r = lane; r < d.n_rows; r += 32) {  // one 2*HD-byte copy per row
                 const int item_row = d.row0 + r;
-                const int occ = a.occ[d.occ_off + item_row / g];
+                int occ = a.occ[d.occ_off + item_row / g];
+                if (!check(in_range(occ, a.ext.n), a.err)) occ = 0;
                 const uint16_t* src = a.q + ((int64_t)occ * a.hq + d.kvh * g + item_row % g) * HD;
                 bulk_g2s(smem_u32(qbuf + r * Smem<HD>::kQPitch), src, HD * 2, smem_u32(&c.qfull));
             }
@@ -1455,6 +1486,17 @@ __device__ void tc_fetch(const DecodeArgs& a, CtlTc& c, uint8_t* qbuf) {
         const int word = (u >= 0 && lane < kUnitWords) ? a.units[(int64_t)u * kUnitWords + lane] : 0;
         const int n_tiles = __shfl_sync(0xffffffffu, word, U_N_TILES);
         const int tile_off = __shfl_sync(0xffffffffu, word, U_TILE_OFF);
+        if constexpr (kBoundsCheck) {
+            const int w_occ = __shfl_sync(0xffffffffu, word, U_OCC_OFF), w_row0 = __shfl_sync(0xffffffffu, word, U_ROW0);
+            const int w_rows = __shfl_sync(0xffffffffu, word, U_N_ROWS);
+            const int w_slot = __shfl_sync(0xffffffffu, word, U_SLOT_BASE), w_kvh = __shfl_sync(0xffffffffu, word, U_KVH);
+            const int w_kind = __shfl_sync(0xffffffffu, word, U_KIND);
+            if (u >= 0 && !(w_kind == KIND_TC && unit_ok(tile_off, n_tiles, w_occ, w_row0, w_rows, w_slot, w_kvh,
+                                                         kTcRowsPerUnit, a.vis != nullptr, a.ext))) {
+                if (lane == 0) atomicOr(a.err, kErrBounds);  // a bad unit record: this CTA takes no more units
+                u = -1;
+            }
+        }
         if (u >= 0)
             for (int t = lane; t < n_tiles; t += 32) c.tiles[q][t] = a.tiles[tile_off + t];
         if (lane < kUnitWords) reinterpret_cast<volatile int*>(c.desc[q])[lane] = word;
@@ -1486,7 +1528,8 @@ __device__ void tc_fetch(const DecodeArgs& a, CtlTc& c, uint8_t* qbuf) {
         for (int i = 0; i < kRowsPerLane; ++i) {
             const int r = lane + 32 * i;
             const int item_row = row0 + r, p = item_row / g, hh = item_row - p * g;
-            const int occ = r >= n_rows ? 0 : in_order ? occ_off + p : a.occ[occ_off + p];
+            int occ = r >= n_rows ? 0 : in_order ? occ_off + p : a.occ[occ_off + p];
+            if (!check(in_range(occ, a.ext.n), a.err)) occ = 0;
             src_off[i] = ((int64_t)occ * a.hq + kvh * g + hh) * HD;
         }
         const uint32_t q_base = smem_u32(qbuf);
@@ -1515,7 +1558,7 @@ __device__ __forceinline__ void issue_half(const DecodeArgs& a, int kvh, int kv,
     uint32_t bytes = 0;
     int valid[2] = {0, 0};
     for (int j = 0; j < 2; ++j)
-        if (w[j] >= 0) {
+        if (w[j] >= 0 && check(tile_word_ok(w[j], a.ext.pool_blocks), a.err)) {  // a bad word: a missing tile
             valid[j] = (w[j] & ((1 << kTileValidBits) - 1)) + 1;
             bytes += (uint32_t)(valid[j] * HD * 2);
         }
@@ -1719,11 +1762,18 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
         const int n_pairs = (d.n_tiles + 1) / 2;
         float m_used = -INFINITY, l = 0.f;
         int vis = 0x7fffffff, pos = d.pos0;
-        if (CAUSAL && row < d.n_rows) vis = a.vis[a.occ[d.occ_off + (d.row0 + row) / a.group]];
+        if (CAUSAL && row < d.n_rows) {
+            const int occ = a.occ[d.occ_off + (d.row0 + row) / a.group];
+            vis = check(in_range(occ, a.ext.n), a.err) ? a.vis[occ] : 0;
+        }
         for (int j = 0; j < n_pairs; ++j) {
             const uint32_t g_stage = gs + j, sb = g_stage & 1;
-            const int v0 = (tw[2 * j] & ((1 << kTileValidBits) - 1)) + 1;
-            const int v1 = 2 * j + 1 < d.n_tiles ? (tw[2 * j + 1] & ((1 << kTileValidBits) - 1)) + 1 : 0;
+            int v0 = (tw[2 * j] & ((1 << kTileValidBits) - 1)) + 1;
+            int v1 = 2 * j + 1 < d.n_tiles ? (tw[2 * j + 1] & ((1 << kTileValidBits) - 1)) + 1 : 0;
+            if (kBoundsCheck) {  // a tile the streamer refused holds no token
+                if (!tile_word_ok(tw[2 * j], a.ext.pool_blocks)) v0 = 0;
+                if (v1 && !tile_word_ok(tw[2 * j + 1], a.ext.pool_blocks)) v1 = 0;
+            }
             // CAUSAL: tokens of tile h visible to this row: lim_h = min(valid, vis - position)
             int lim0 = v0, lim1 = v1;
             if (CAUSAL) {
@@ -1844,7 +1894,7 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
             }
             continue;
         }
-        const bool live = row < d.n_rows;
+        bool live = row < d.n_rows;
         const bool final_out = CAUSAL && d.slot_base < 0;  // the row's only unit: final O and LSE
         float* dst = nullptr;
         uint16_t* dst16 = nullptr;
@@ -1853,8 +1903,9 @@ __device__ void tc_consume(const DecodeArgs& a, CtlTc& c) {
             const int qh = d.kvh * a.group + item_row % a.group;
             if (final_out) {
                 const int occ = a.occ[d.occ_off + item_row / a.group];
+                live = check(in_range(occ, a.ext.n), a.err);
                 dst16 = a.out + ((int64_t)occ * a.hq + qh) * HD;
-                a.out_lse[(int64_t)occ * a.hq + qh] = (m_used + __log2f(l)) * 0.69314718055994531f;
+                if (live) a.out_lse[(int64_t)occ * a.hq + qh] = (m_used + __log2f(l)) * 0.69314718055994531f;
             } else {
                 const int slot = d.slot_base + item_row / a.group;
                 dst = a.part_o + ((int64_t)slot * a.hq + qh) * HD;
@@ -1976,6 +2027,7 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
     if (warp_global >= a.n * a.hq) return;
     const int i = warp_global / a.hq, qh = warp_global % a.hq;
     const int beg = a.merge_off[i], ns = a.merge_off[i + 1] - beg;
+    if (!check(merge_range_ok(beg, beg + ns, a.n_merge) && (ns == 0 || a.n_slots > 0), a.err)) return;
     if (ns == 0) return;  // written directly by its only unit
     float acc[DPL];
 #pragma unroll
@@ -1990,7 +2042,10 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
         float lse = -INFINITY;
         if (k < ns) {
             slot = a.merge_slot[beg + k];
-            lse = a.part_lse[(int64_t)slot * a.hq + qh];
+            if (check(in_range(slot, a.n_slots), a.err))
+                lse = a.part_lse[(int64_t)slot * a.hq + qh];
+            else
+                slot = 0;  // weight 0, a valid row to read
         }
         float cm = lse;
 #pragma unroll
@@ -2219,8 +2274,9 @@ cudaError_t launch_wait_probe(int32_t* err, uint64_t limit_ns, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_patch(int32_t* sched, const int32_t* pairs, int32_t n, cudaStream_t s) {
-    patch_kernel<<<(n + 255) / 256, 256, 0, s>>>(sched, pairs, n);
+cudaError_t launch_patch(int32_t* sched, const int32_t* pairs, int32_t n, cudaStream_t s, int64_t sched_words,
+                         int32_t* err) {
+    patch_kernel<<<(n + 255) / 256, 256, 0, s>>>(sched, pairs, n, sched_words, err);
     return cudaGetLastError();
 }
 
