@@ -5,7 +5,11 @@ forest shaped like TreePO rollouts (all rows of the hot path: tree-walk
 schedule -> split-KV attention over shared path segments -> LSE merge).
 Inputs (pool K/V, Q) are resident in HBM when the timed region starts; the
 unique KV read per step (>= 1.8 GB for the full workloads) is far larger
-than L2 (129 MB), so no flush is needed between steps.
+than L2 (129 MB), so no flush is needed between steps. The K timed calls
+run as a user makes them; the same K calls then run again with every call's
+kernels bracketed by CUDA events on the tree's stream, which gives the kernel
+durations the roofline divides by (the brackets themselves cost a call a few
+microseconds, so the rate comes from the first region).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # the CPU oracle, timed on host cores
@@ -433,7 +437,6 @@ def bench_rollout(args):
         forest.rollout(params(w))
     forest.sync()
     sampler = _clocks_start()
-    tp.tp_profile_start(forest.handle)
     t0 = time.perf_counter()
     stats, algo_bytes, rows = [], 0, 0
     for k in range(args.steps):
@@ -444,6 +447,12 @@ def bench_rollout(args):
         rows += r
     forest.sync()
     wall = time.perf_counter() - t0
+    # the same rollouts again with every kernel bracketed by CUDA events: the
+    # kernel times (the brackets cost each of the thousands of small calls a
+    # few microseconds, so the rate comes from the region above)
+    tp.tp_profile_start(forest.handle)
+    for k in range(args.steps):
+        forest.rollout(params(args.warmup + k))
     kt = tp.tp_profile_stop(forest.handle)
     clocks = sampler.stop()
     tokens = sum(st["tokens"] for st in stats)
@@ -470,6 +479,7 @@ def bench_rollout(args):
                      "algorithmic_bytes_per_step": algo_bytes / args.steps,
                      "peak_source": f"{kind} hbm_gbs"},
         "kernel_ms_per_step": {k: v["ms"] / args.steps for k, v in kt.items()},
+        "kernel_times": "CUDA events around every kernel, over a second run of the same rollouts",
         "host_ms_per_step": (wall * 1e3 - sum(v["ms"] for v in kt.values())) / args.steps,
         "e2e": {"value": tokens / wall, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0,
                 "note": "the rollout is host-driven end to end: value is already wall-clock through tp_rollout"},
@@ -794,17 +804,24 @@ def main():
             dist.barrier()
         return a.elapsed_time(b)
 
-    # ---- warm-up, then the timed region (kernel times recorded live)
+    # ---- warm-up, then the timed region: K calls as a user makes them
     steps(args.warmup, args.flags)
     torch.cuda.synchronize()
     sampler = _clocks_start(lambda: steps(1, args.flags), device=local)
-    tp.tp_profile_start(forest.handle)
     ms_total = timed(args.steps, args.flags)
+    # ---- the same K calls with each call's kernels bracketed by CUDA events
+    # on the tree's stream (its attention kernels together, the merge alone):
+    # the kernel durations the roofline divides by, measured live. The
+    # brackets cost a call a few microseconds, so `value` comes from the
+    # region above, not from this one.
+    tp.tp_profile_start(forest.handle)
+    ms_profiled = timed(args.steps, args.flags)
     ktimes = tp.tp_profile_stop(forest.handle)
     clocks = sampler.stop()
     forest.sync()
 
-    # ---- controls: schedule rebuilt every call, and no prefix sharing
+    # ---- controls, timed like the first region: schedule rebuilt every
+    # call, and no prefix sharing
     ms_uncached = timed(args.steps, args.flags | tp.TP_DECODE_NO_CACHE)
     steps(2, tp.TP_DECODE_NO_SHARE)
     ms_noshare = timed(args.steps, tp.TP_DECODE_NO_SHARE)
@@ -833,8 +850,8 @@ def main():
     e2e_sync_s = time.perf_counter() - t0
 
     # ---- max over ranks
-    ms_total, ms_uncached, ms_noshare, e2e_s, e2e_sync_s = max_over_ranks(
-        [ms_total, ms_uncached, ms_noshare, e2e_s, e2e_sync_s], dev)
+    ms_total, ms_profiled, ms_uncached, ms_noshare, e2e_s, e2e_sync_s = max_over_ranks(
+        [ms_total, ms_profiled, ms_uncached, ms_noshare, e2e_s, e2e_sync_s], dev)
     leaves_all = n * world
 
     if rank == 0:
@@ -844,6 +861,7 @@ def main():
         dec = ktimes["decode"]
         mer = ktimes["merge"]
         dec_ms = dec["ms"] / args.steps  # one bracket per call around its concurrent attention kernels
+        assert dec["launches"] > 0 and dec_ms * args.steps <= ms_profiled * 1.001
         algo_dec = desc["unique_kv_bytes"] + desc["q_bytes"]
         achieved = algo_dec / (dec_ms / 1e3) / 1e9
         call_bytes = desc["unique_kv_bytes"] + desc["q_bytes"] + desc["o_bytes"] + desc["lse_bytes"]
@@ -863,10 +881,13 @@ def main():
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic, "kernel": "decode_kernel",
                          "algorithmic_bytes_per_launch": algo_dec, "launch_ms": dec_ms,
+                         "measured": "CUDA events around each call's attention kernels on the tree's stream, over "
+                                     "a second timed region of the same K calls",
                          "peak_source": f"{peak_kind} hbm_gbs"},
             "call_roofline": {"bytes": call_bytes, "achieved": call_gbs, "frac": call_gbs / peak,
                               "note": "unique KV + Q + O + LSE per tp_decode call / ms_per_step"},
             "kernel_ms_per_step": {"decode": dec_ms, "merge": mer["ms"] / args.steps},
+            "ms_per_step_profiled": ms_profiled / args.steps,
             "ms_per_step_schedule_uncached": ms_uncached / args.steps,
             "no_share_ms_per_step": ms_noshare / args.steps,
             "sharing_speedup": ms_noshare / ms_total,

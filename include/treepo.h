@@ -185,7 +185,10 @@ tp_status tp_decode(tp_tree* tree, const tp_node* leaves, int32_t n, const void*
 #define TP_DECODE_ALL_TCGEN05 16u     /* the default: every unit of > 16 stacked     */
                                       /* rows on tcgen05 (128-row units, running     */
                                       /* concurrently with the mma.sync units of one */
-                                      /* 16-row tile; measured fastest on GB300)     */
+                                      /* 16-row tile; measured fastest on GB300);    */
+                                      /* by default a call reading < 1 MiB of K/V    */
+                                      /* runs all on mma.sync (one kernel: latency-  */
+                                      /* bound), this flag forces tcgen05 there too  */
 #define TP_MMA_SYNC 32u               /* no tcgen05: stacked rows on mma.sync in     */
                                       /* 64-row units (decode and tp_prefill)        */
 tp_status tp_decode_ex(tp_tree* tree, const tp_node* leaves, int32_t n, const void* Q, void* O,

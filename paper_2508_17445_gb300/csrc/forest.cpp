@@ -132,10 +132,6 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     const int32_t hq = t->cfg.num_q_heads, hkv = t->cfg.num_kv_heads, g = hq / hkv;
     const bool share = !(flags & TP_DECODE_NO_SHARE);
     const bool cuda_core_small = (flags & TP_DECODE_CUDA_CORE_SMALL) != 0;
-    // tcgen05 for every unit of more than one 16-row MMA tile unless
-    // TP_MMA_SYNC; TP_DECODE_TCGEN05 alone keeps it to long, tall chunks
-    const bool use_tc = (flags & TP_MMA_SYNC) == 0;
-    const bool all_tc = use_tc && !((flags & TP_DECODE_TCGEN05) && !(flags & TP_DECODE_ALL_TCGEN05));
     for (int32_t i = 0; i < n; ++i) {
         tp_status st = check_live(t, leaves[i], true);
         if (st != TP_OK) return st;
@@ -260,6 +256,16 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     for (const Item& it : items) work += (int64_t)it.n_tiles * hkv;
     const int32_t chunk = (int32_t)std::min<int64_t>(
         kMaxChunkTiles, std::max<int64_t>(kMinChunkTiles, (work + kTargetUnits - 1) / kTargetUnits));
+    // tcgen05 for every unit of more than one 16-row MMA tile unless
+    // TP_MMA_SYNC; TP_DECODE_TCGEN05 alone keeps it to long, tall chunks. A
+    // call reading less than kSmallCallBytes of K/V is bound by launch
+    // latency: its stacked rows stay on mma.sync, so the whole call is one
+    // attention kernel on the tree's stream, without the tcgen05 kernel's
+    // side-stream fork and join (TP_DECODE_ALL_TCGEN05 still forces tcgen05).
+    const int64_t tile_bytes = (int64_t)t->cfg.block_tokens * t->cfg.head_dim * 2 * 2;
+    const bool small_call = work * tile_bytes < kSmallCallBytes && !(flags & TP_DECODE_ALL_TCGEN05);
+    const bool use_tc = (flags & TP_MMA_SYNC) == 0 && !small_call;
+    const bool all_tc = use_tc && !((flags & TP_DECODE_TCGEN05) && !(flags & TP_DECODE_ALL_TCGEN05));
 
     // 5. units, partial slots and merge entries
     std::vector<int32_t>& tc_units = X.units[0];

@@ -37,6 +37,9 @@ constexpr int kTcMinRows = 64;
 constexpr int kTcMinTiles = 32;
 constexpr int kTcAnyRows = 17;
 constexpr int kTcRowsPerUnit = 128;
+// Decode calls reading less K/V than this (about a microsecond of HBM time)
+// keep every unit on mma.sync: one attention kernel, no side stream.
+constexpr int64_t kSmallCallBytes = 1 << 20;
 // Longest unit in pool blocks (the decode kernel keeps a unit's tile words
 // in shared memory).
 constexpr int kMaxUnitTiles = 128;

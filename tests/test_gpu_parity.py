@@ -101,7 +101,9 @@ def run_and_compare(script, flags=0, sample=None, leaves=None, q=None):
     return O, LSE, err
 
 
-FLAG_SETS = [0, tp.TP_DECODE_CUDA_CORE_SMALL, tp.TP_DECODE_NO_SHARE, tp.TP_MMA_SYNC]
+# default routing, CUDA-core small units, no sharing, all mma.sync, and
+# tcgen05 forced (calls under 1 MiB of K/V default to mma.sync only)
+FLAG_SETS = [0, tp.TP_DECODE_CUDA_CORE_SMALL, tp.TP_DECODE_NO_SHARE, tp.TP_MMA_SYNC, tp.TP_DECODE_ALL_TCGEN05]
 
 
 # --------------------------------------------------------------------------
@@ -119,6 +121,7 @@ def test_random_forests(seed, heads):
     s = workloads.random_tree(seed=seed, heads=heads, n_prompts=3, max_depth=5,
                               prompt_range=(1, 400), seg_range=(1, 200))
     run_and_compare(s, flags=FLAG_SETS[seed % 4])
+    run_and_compare(s, flags=tp.TP_DECODE_ALL_TCGEN05)
 
 
 @pytest.mark.parametrize("heads", [workloads.Heads(32, 2, 64), workloads.Heads(24, 2, 128)])

@@ -287,7 +287,17 @@ def check_schedule(f, ids, model, script, leaves_sid, flags=0):
     leaves = [ids[x] for x in leaves_sid]
     S = tp.tp_debug_schedule(f.handle, leaves, flags)
     assert S["group"] == g
-    all_tc = not flags & tp.TP_MMA_SYNC and not (flags & tp.TP_DECODE_TCGEN05 and not flags & tp.TP_DECODE_ALL_TCGEN05)
+    # a call reading less than 1 MiB of K/V (its path blocks, counted whole:
+    # each shared block once, or once per leaf without sharing) keeps every
+    # unit on mma.sync unless tcgen05 is forced
+    nodes = [x for x in {y for lf in leaves_sid for y in model.path_nodes(lf)}] if not flags & tp.TP_DECODE_NO_SHARE \
+        else [y for lf in leaves_sid for y in model.path_nodes(lf)]
+    blocks = sum(-(-model.nodes[x].n_tokens // BT) for x in nodes)
+    small = blocks * heads.num_kv_heads * BT * heads.head_dim * 4 < (1 << 20) and not flags & tp.TP_DECODE_ALL_TCGEN05
+    all_tc = not flags & tp.TP_MMA_SYNC and not small and not (
+        flags & tp.TP_DECODE_TCGEN05 and not flags & tp.TP_DECODE_ALL_TCGEN05)
+    if small:
+        assert S["n_tc_units"] == 0
     covered = collections.defaultdict(list)
     slots_of = collections.defaultdict(set)
     chunk_reads = collections.Counter()
@@ -304,7 +314,7 @@ def check_schedule(f, ids, model, script, leaves_sid, flags=0):
             if flags & tp.TP_DECODE_CUDA_CORE_SMALL:
                 assert nrows >= 16 or row0 > 0
         else:                              # tcgen05: stacked rows in 128-row blocks
-            assert kind == 2 and not flags & tp.TP_MMA_SYNC
+            assert kind == 2 and not flags & tp.TP_MMA_SYNC and not small
             assert 1 <= nrows <= 128
             if all_tc:
                 assert row0 > 0 or nrows >= 17
