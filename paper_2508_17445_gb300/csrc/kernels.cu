@@ -581,7 +581,18 @@ struct Smem {
     static constexpr int kQPitch = HD * 2 + 16;
     static constexpr int kQBytes = kConsumerWarps * 16 * kQPitch;
     static constexpr int kBytes = kRingBytes + kParkFloats * 4 + kQBytes;
+    // the CUDA-core kind stages no query rows and combines through a smaller
+    // park (per warp: 8 maxima, 8 sums, 8 rows of HD), followed by its score
+    // scratch ([warp][64 tokens][8 rows]); at ~90 KB two CTAs share an SM
+    static constexpr int kCcParkFloats = kConsumerWarps * 8 * (2 + HD);
+    static constexpr int kCcScratchFloats = kConsumerWarps * kStageTokens * 8;
+    static constexpr int kCcBytes = kRingBytes + (kCcParkFloats + kCcScratchFloats) * 4;
 };
+
+template <int HD, int KIND>
+constexpr int decode_smem() {
+    return KIND == KIND_CUDA_CORE ? Smem<HD>::kCcBytes : Smem<HD>::kBytes;
+}
 
 // Shared control block of one CTA.
 struct Ctl {
@@ -751,7 +762,8 @@ struct CudaCorePath {
         const int TW = kStageTokens / n_sp;  // tokens of a stage this warp handles
         const int dg = lane % LPT, ts = lane / LPT;
 
-        // q rows of this warp, 8 dims per lane, pre-scaled to the log2 domain
+        // q rows of this warp, 8 dims per lane, pre-scaled to the log2 domain;
+        // packed in row pairs (rows 2i, 2i + 1) for the f32x2 dot products
         float qf[NR][8];
 #pragma unroll
         for (int r = 0; r < NR; ++r) {
@@ -773,11 +785,17 @@ struct CudaCorePath {
                 for (int k = 0; k < 8; ++k) qf[r][k] = 0.f;
             }
         }
-        float o[NR][8];
+        uint64_t q2[NR / 2][8];
+#pragma unroll
+        for (int i = 0; i < NR / 2; ++i)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) q2[i][k] = f2_pack(qf[2 * i][k], qf[2 * i + 1][k]);
+        // o of each row in dimension pairs (k, k + 1)
+        uint64_t o2[NR][4];
 #pragma unroll
         for (int r = 0; r < NR; ++r)
 #pragma unroll
-            for (int k = 0; k < 8; ++k) o[r][k] = 0.f;
+            for (int k = 0; k < 4; ++k) o2[r][k] = 0ull;
         // running max / sum of row (lane >> 2), replicated over its quad
         float m_run = -INFINITY, l_run = 0.f;
         float* sc = scratch + warp * (kStageTokens * NR);  // [token][row]
@@ -793,20 +811,23 @@ struct CudaCorePath {
                 const int t = tbase + s0 + ts;  // token within the stage
                 const uint4 kw = *reinterpret_cast<const uint4*>(sk + kv_off<kStageTokens>(t, dg));
                 const uint32_t kk[4] = {kw.x, kw.y, kw.z, kw.w};
-                float kf[8];
+                // two rows per f32x2 FMA; each row's sum in the same order
+                // (and rounding) as a scalar fmaf chain over k
+                uint64_t acc2[NR / 2];
+#pragma unroll
+                for (int i = 0; i < NR / 2; ++i) acc2[i] = 0ull;
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
-                    kf[2 * k] = bf_lo(kk[k]);
-                    kf[2 * k + 1] = bf_hi(kk[k]);
+                    const float k0 = bf_lo(kk[k]), k1 = bf_hi(kk[k]);
+                    const uint64_t kb0 = f2_pack(k0, k0), kb1 = f2_pack(k1, k1);
+#pragma unroll
+                    for (int i = 0; i < NR / 2; ++i) acc2[i] = f2_fma(q2[i][2 * k], kb0, acc2[i]);
+#pragma unroll
+                    for (int i = 0; i < NR / 2; ++i) acc2[i] = f2_fma(q2[i][2 * k + 1], kb1, acc2[i]);
                 }
                 float acc[NR];
 #pragma unroll
-                for (int r = 0; r < NR; ++r) {
-                    float x = 0.f;
-#pragma unroll
-                    for (int k = 0; k < 8; ++k) x = fmaf(qf[r][k], kf[k], x);
-                    acc[r] = x;
-                }
+                for (int i = 0; i < NR / 2; ++i) f2_unpack(acc2[i], acc[2 * i], acc[2 * i + 1]);
                 float s = transpose_reduce(acc, lane);
                 const int valid = (t & 31) < ((t < kBlockTokens) ? v0 : v1);
                 if (!valid) s = -INFINITY;
@@ -838,34 +859,40 @@ struct CudaCorePath {
             __syncwarp();
             // ---- rescale and accumulate P.V
             if (!__all_sync(0xffffffffu, alpha == 1.f)) {
+                const uint64_t nz = f2_pack(-0.f, -0.f);  // x * al + (-0) = x * al exactly
 #pragma unroll
                 for (int r = 0; r < NR; ++r) {
                     const float al = __shfl_sync(0xffffffffu, alpha, r * 4);
+                    const uint64_t al2 = f2_pack(al, al);
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) o[r][k] *= al;
+                    for (int k = 0; k < 4; ++k) o2[r][k] = f2_fma(o2[r][k], al2, nz);
                 }
             }
             for (int s0 = 0; s0 < TW; s0 += TPS) {
                 const int t = tbase + s0 + ts;
                 const uint4 vw = *reinterpret_cast<const uint4*>(sv + kv_off<kStageTokens>(t, dg));
                 const uint32_t vv[4] = {vw.x, vw.y, vw.z, vw.w};
-                float vf[8];
+                uint64_t v2[4];  // dimension pairs (2k, 2k + 1)
 #pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    vf[2 * k] = bf_lo(vv[k]);
-                    vf[2 * k + 1] = bf_hi(vv[k]);
-                }
+                for (int k = 0; k < 4; ++k) v2[k] = f2_pack(bf_lo(vv[k]), bf_hi(vv[k]));
                 const float4 p0 = *reinterpret_cast<const float4*>(&sc[(s0 + ts) * NR]);
                 const float4 p1 = *reinterpret_cast<const float4*>(&sc[(s0 + ts) * NR + 4]);
                 const float p[NR] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
 #pragma unroll
-                for (int r = 0; r < NR; ++r)
+                for (int r = 0; r < NR; ++r) {
+                    const uint64_t pb = f2_pack(p[r], p[r]);
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) o[r][k] = fmaf(p[r], vf[k], o[r][k]);
+                    for (int k = 0; k < 4; ++k) o2[r][k] = f2_fma(pb, v2[k], o2[r][k]);
+                }
             }
             __syncwarp();  // sc is rewritten by the next stage's scores
             rr.release(lane);
         }
+        float o[NR][8];
+#pragma unroll
+        for (int r = 0; r < NR; ++r)
+#pragma unroll
+            for (int k = 0; k < 4; ++k) f2_unpack(o2[r][k], o[r][2 * k], o[r][2 * k + 1]);
         // ---- fold the TPS token slots of each lane column
 #pragma unroll
         for (int off = LPT; off < 32; off <<= 1)
@@ -1284,10 +1311,10 @@ template <int HD, int KIND>
 __global__ void __launch_bounds__(kDecodeThreads, 2) decode_kernel(const DecodeArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(16) Ctl ctl;
-    __shared__ __align__(16) float cc_scratch[KIND == KIND_CUDA_CORE ? kConsumerWarps * kStageTokens * 8 : 4];
     uint8_t* ring = smem;
     float* park = reinterpret_cast<float*>(smem + Smem<HD>::kRingBytes);
-    uint8_t* qbuf = smem + Smem<HD>::kRingBytes + Smem<HD>::kParkFloats * 4;
+    uint8_t* qbuf = smem + Smem<HD>::kRingBytes + Smem<HD>::kParkFloats * 4;  // tensor kinds only
+    float* cc_scratch = park + Smem<HD>::kCcParkFloats;                         // CUDA-core kind only
     const int tid = threadIdx.x, warp = tid >> 5;
     // zero the ring once: rows past a partial block are never copied and must
     // hold finite values (their probabilities are exactly 0)
@@ -2133,10 +2160,10 @@ int decode_grid() {
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         if (cudaFuncSetAttribute(decode_kernel<HD, KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 Smem<HD>::kBytes) != cudaSuccess)
+                                 decode_smem<HD, KIND>()) != cudaSuccess)
             return 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_kernel<HD, KIND>, kDecodeThreads,
-                                                          Smem<HD>::kBytes) != cudaSuccess)
+                                                          decode_smem<HD, KIND>()) != cudaSuccess)
             return 0;
         return sms * std::max(per_sm, 1);
     }();
@@ -2151,7 +2178,7 @@ cudaError_t launch_range(DecodeArgs a, int begin, int end, int32_t* counter, cud
     a.unit_begin = begin;
     a.unit_end = end;
     a.counter = counter;
-    decode_kernel<HD, KIND><<<std::min(end - begin, slots), kDecodeThreads, Smem<HD>::kBytes, s>>>(a);
+    decode_kernel<HD, KIND><<<std::min(end - begin, slots), kDecodeThreads, decode_smem<HD, KIND>(), s>>>(a);
     return cudaGetLastError();
 }
 
