@@ -2123,22 +2123,34 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
 #pragma unroll
                 for (int u = 0; u < 4; ++u) l2_discard(srcs[u]);
         }
-        for (; j < cnt; ++j) {
-            const int64_t sl = __shfl_sync(0xffffffffu, slot, j);
-            const float wj = __shfl_sync(0xffffffffu, w, j);
-            const float* src = a.part_o + (sl * a.hq + qh) * HD + lane * DPL;
-            float xs[DPL];
-            if constexpr (DPL == 4) {
-                const float4 v = ld_f4_hint(src, pol);
-                xs[0] = v.x, xs[1] = v.y, xs[2] = v.z, xs[3] = v.w;
-            } else {
-                const float2 v = ld_f2_hint(src, pol);
-                xs[0] = v.x, xs[1] = v.y;
+        if (j < cnt) {  // the last 1-3 rows as one batch, all loads in flight together
+            float wj[4];
+            float x[4][DPL];
+            const float* srcs[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const bool on = j + u < cnt;
+                const int64_t sl = __shfl_sync(0xffffffffu, slot, on ? j + u : j);  // off: re-read row j, weight 0
+                wj[u] = __shfl_sync(0xffffffffu, w, on ? j + u : j) * (on ? 1.f : 0.f);
+                const float* src = a.part_o + (sl * a.hq + qh) * HD + lane * DPL;
+                srcs[u] = on ? src : nullptr;
+                if constexpr (DPL == 4) {
+                    const float4 v = ld_f4_hint(src, pol);
+                    x[u][0] = v.x, x[u][1] = v.y, x[u][2] = v.z, x[u][3] = v.w;
+                } else {
+                    const float2 v = ld_f2_hint(src, pol);
+                    x[u][0] = v.x, x[u][1] = v.y;
+                }
             }
 #pragma unroll
-            for (int d = 0; d < DPL; ++d) acc[d] += wj * xs[d];
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int d = 0; d < DPL; ++d) acc[d] += wj[u] * x[u][d];
             __syncwarp();
-            if (line_lead) l2_discard(src);
+            if (line_lead)
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (srcs[u]) l2_discard(srcs[u]);
         }
     }
     const float inv = 1.f / L;
