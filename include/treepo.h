@@ -549,14 +549,17 @@ tp_status tp_debug_gather(tp_tree* tree, tp_node leaf, void* K_out, void* V_out,
  *   [0] magic 0x54505344, [1] n_units, [2] n_tiles, [3] n_occ_entries,
  *   [4] n (leaf occurrences), [5] n_slots, [6] n_merge_entries, [7] group g,
  *   [8] n_mma_units, [9] n_tcgen05_units, [10] 0 (1 for prefill schedules),
- *   [11..15] reserved (0),
+ *   [11] 16 (words per merge record), [12..15] reserved (0),
  *   then units  [n_units][8]: tile_off, n_tiles, occ_off, row0, n_rows,
  *                             slot_base, kv_head, kind (0 CUDA-core,
  *                             1 mma.sync, 2 tcgen05); tcgen05 units first,
  *                             then mma.sync, then CUDA-core,
  *   then tiles  [n_tiles]: block << 7 | (valid_tokens - 1),
  *   then occ    [n_occ_entries]: leaf occurrence index (row i of Q),
- *   then merge_off [n + 1], then merge_slot [n_merge_entries].
+ *   then merge_off [n + 1], then merge_slot [n_merge_entries],
+ *   then merge_rec [n][16]: occurrence i's slot count and its slots in
+ *                             merge_slot order, zero-padded ([-1, 0...] when
+ *                             it has more than 15: the CSR holds them).
  * Unit row r (0 <= r < n_rows) is item row row0 + r = p * g + j: occurrence
  * occ[occ_off + p], q-head kv_head * g + j, written to partial slot
  * slot_base + p. Occurrence i merges slots merge_slot[merge_off[i] ..
@@ -574,8 +577,10 @@ tp_status tp_debug_schedule(tp_tree* tree, const tp_node* leaves, int32_t n, uin
  * their partial slots below n_slots (slot_base -1 only in prefill
  * schedules), its kv head below num_kv_heads; each tile word's block below
  * the tree's pool_blocks with 1..32 valid tokens; each occurrence entry
- * below n; each occurrence's merge range inside the merge list; each merge
- * slot below n_slots. violations: host int64 [5] receives the number of bad
+ * below n; each occurrence's merge range inside the merge list, and its
+ * merge record's count equal to the range's length (or -1 past 15); each
+ * merge slot, and each slot of a merge record, below n_slots (a record's
+ * slots equal to its CSR range). violations: host int64 [5] receives the number of bad
  * unit records, tile words, occurrence entries, merge ranges and merge
  * slots. Errors: TP_ERR_INVALID_ARG (not a schedule: bad magic, bad header,
  * shorter than its header says).
@@ -583,7 +588,7 @@ tp_status tp_debug_schedule(tp_tree* tree, const tp_node* leaves, int32_t n, uin
 tp_status tp_debug_check_schedule(tp_tree* tree, const int32_t* words, int64_t n_words, int64_t* violations);
 
 /* The schedule tp_prefill would run, in the layout above with header word
- * [10] = 1 and two more sections at the end: unit_pos [n_units] (path
+ * [10] = 1 and two more sections before merge_rec: unit_pos [n_units] (path
  * position of each unit's first token) and vis [n] (tokens of its path that
  * occurrence i -- query token i -- may see). Occurrences are the query
  * tokens; units are tcgen05 units (mma.sync units with TP_MMA_SYNC); a unit

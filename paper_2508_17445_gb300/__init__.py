@@ -349,6 +349,9 @@ def _parse_schedule(w: np.ndarray) -> Dict[str, np.ndarray]:
     if w[10] == 1:
         out["unit_pos"] = w[off: off + n_units]
         out["vis"] = w[off + n_units: off + n_units + n]
+        off += n_units + n
+    rw = int(w[11])
+    out["merge_rec"] = w[off: off + n * rw].reshape(n, rw)
     return out
 
 

@@ -809,6 +809,7 @@ tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O
     tp::MergeArgs m;
     m.merge_off = t->d_sched + S.off_merge_off;
     m.merge_slot = t->d_sched + S.off_merge_slot;
+    m.merge_rec = t->d_sched + S.off_merge_rec;
     m.part_o = a.part_o;
     m.part_lse = a.part_lse;
     m.out = (uint16_t*)O;
@@ -896,6 +897,7 @@ tp_status tp_decode_noalloc(tp_tree* t, const tp_node* leaves, int32_t n, const 
     tp::MergeArgs m;
     m.merge_off = d_sched + S.off_merge_off;
     m.merge_slot = d_sched + S.off_merge_slot;
+    m.merge_rec = d_sched + S.off_merge_rec;
     m.part_o = a.part_o;
     m.part_lse = a.part_lse;
     m.out = (uint16_t*)O;
@@ -1074,7 +1076,9 @@ tp_status tp_debug_check_schedule(tp_tree* t, const int32_t* w, int64_t n_words,
         return fail(t, TP_ERR_INVALID_ARG, "bad schedule header");
     const int64_t off_units = tp::kSchedHeaderWords, off_tiles = off_units + (int64_t)n_units * tp::kUnitWords;
     const int64_t off_occ = off_tiles + n_tiles, off_moff = off_occ + n_occ, off_mslot = off_moff + n + 1;
-    const int64_t end = off_mslot + n_merge + (prefill ? (int64_t)n_units + n : 0);
+    const int64_t off_mrec = off_mslot + n_merge + (prefill ? (int64_t)n_units + n : 0);
+    if (w[11] != tp::kMergeRecWords) return fail(t, TP_ERR_INVALID_ARG, "bad schedule header (merge records)");
+    const int64_t end = off_mrec + (int64_t)n * tp::kMergeRecWords;
     if (n_words < end) return fail(t, TP_ERR_INVALID_ARG, "schedule shorter than its header says");
     tp::Extents x;
     x.pool_blocks = t->cfg.pool_blocks;
@@ -1098,6 +1102,18 @@ tp_status tp_debug_check_schedule(tp_tree* t, const int32_t* w, int64_t n_words,
     for (int64_t k = 0; k < n_occ; ++k) bad[2] += !tp::in_range(w[off_occ + k], n);
     for (int32_t i = 0; i < n; ++i) bad[3] += !tp::merge_range_ok(w[off_moff + i], w[off_moff + i + 1], n_merge);
     for (int64_t k = 0; k < n_merge; ++k) bad[4] += !tp::in_range(w[off_mslot + k], n_slots);
+    // merge records: the count of the CSR range (or -1 past 15) and its slots
+    for (int32_t i = 0; i < n; ++i) {
+        const int32_t* r = w + off_mrec + (int64_t)i * tp::kMergeRecWords;
+        const int64_t beg = w[off_moff + i], cnt = (int64_t)w[off_moff + i + 1] - beg;
+        const bool range_ok = tp::merge_range_ok(w[off_moff + i], w[off_moff + i + 1], n_merge);
+        if (r[0] == -1 ? cnt < tp::kMergeRecWords - 1 : (r[0] < 0 || r[0] >= tp::kMergeRecWords || r[0] != cnt)) {
+            ++bad[3];
+            continue;
+        }
+        for (int32_t k = 0; k < r[0]; ++k)
+            bad[4] += !tp::in_range(r[1 + k], n_slots) || !range_ok || r[1 + k] != w[off_mslot + beg + k];
+    }
     std::memcpy(violations, bad, sizeof bad);
     return TP_OK;
 }

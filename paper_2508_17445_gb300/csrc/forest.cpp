@@ -126,6 +126,22 @@ void merge_csr(SchedScratch& X, int32_t n) {
     for (size_t k = 0; k < X.pair_occ.size(); ++k)
         X.merge_slot[(size_t)X.merge_pos[(size_t)X.pair_occ[k]]++] = X.pair_slot[k];
 }
+
+// Fixed-size merge records from the CSR: [count, slots..., 0...], or
+// [-1, 0...] for an occurrence with more than kMergeRecWords - 1 slots.
+void merge_records(const SchedScratch& X, int32_t n, int32_t* rec) {
+    std::fill(rec, rec + (int64_t)n * kMergeRecWords, 0);
+    for (int32_t i = 0; i < n; ++i) {
+        const int32_t beg = X.merge_off[(size_t)i], cnt = X.merge_off[(size_t)i + 1] - beg;
+        int32_t* r = rec + (int64_t)i * kMergeRecWords;
+        if (cnt >= kMergeRecWords) {
+            r[0] = -1;
+            continue;
+        }
+        r[0] = cnt;
+        std::copy(X.merge_slot.begin() + beg, X.merge_slot.begin() + beg + cnt, r + 1);
+    }
+}
 }  // namespace
 
 tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t flags, Schedule& S) {
@@ -352,7 +368,8 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     S.off_occ = S.off_tiles + S.n_tiles;
     S.off_merge_off = S.off_occ + S.n_occ;
     S.off_merge_slot = S.off_merge_off + n + 1;
-    const int64_t total = S.off_merge_slot + S.n_merge;
+    S.off_merge_rec = S.off_merge_slot + S.n_merge;
+    const int64_t total = S.off_merge_rec + (int64_t)n * kMergeRecWords;
     if (total >= (int64_t)1 << 31) return fail(t, TP_ERR_INVALID_ARG, "schedule too large");
     S.words.resize((size_t)total);
     int32_t* w = S.words.data();
@@ -367,6 +384,7 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     w[7] = g;
     w[8] = S.n_tensor;
     w[9] = S.n_tc;
+    w[11] = kMergeRecWords;
     std::copy(tc_units.begin(), tc_units.end(), w + S.off_units);
     std::copy(tensor_units.begin(), tensor_units.end(), w + S.off_units + tc_units.size());
     std::copy(small_units.begin(), small_units.end(), w + S.off_units + tc_units.size() + tensor_units.size());
@@ -374,6 +392,7 @@ tp_status build_schedule(tp_tree* t, const tp_node* leaves, int32_t n, uint32_t 
     std::copy(occ.begin(), occ.end(), w + S.off_occ);
     std::copy(merge_off.begin(), merge_off.end(), w + S.off_merge_off);
     std::copy(merge_slot.begin(), merge_slot.end(), w + S.off_merge_slot);
+    merge_records(X, n, w + S.off_merge_rec);
     S.leaf_tail.resize(2 * X.tail_node.size());
     for (size_t k = 0; k < X.tail_node.size(); ++k) {
         S.leaf_tail[2 * k] = X.tail_node[k];
@@ -495,7 +514,8 @@ tp_status build_prefill_schedule(tp_tree* t, const tp_node* nodes, const int32_t
     S.off_merge_slot = S.off_merge_off + S.n + 1;
     S.off_unit_pos = S.off_merge_slot + S.n_merge;
     S.off_vis = S.off_unit_pos + S.n_units;
-    const int64_t total = S.off_vis + S.n;
+    S.off_merge_rec = S.off_vis + S.n;
+    const int64_t total = S.off_merge_rec + (int64_t)S.n * kMergeRecWords;
     if (total >= (int64_t)1 << 31) return fail(t, TP_ERR_INVALID_ARG, "schedule too large");
     S.words.resize((size_t)total);
     int32_t* w = S.words.data();
@@ -511,6 +531,7 @@ tp_status build_prefill_schedule(tp_tree* t, const tp_node* nodes, const int32_t
     w[8] = S.n_tensor;
     w[9] = S.n_tc;
     w[10] = 1;  // prefill schedule
+    w[11] = kMergeRecWords;
     for (int32_t k = 0; k < S.n_units; ++k) {
         std::memcpy(w + S.off_units + (int64_t)k * kUnitWords, &recs[(size_t)k * W], sizeof(int32_t) * kUnitWords);
         w[S.off_unit_pos + k] = recs[(size_t)k * W + kUnitWords];
@@ -520,6 +541,7 @@ tp_status build_prefill_schedule(tp_tree* t, const tp_node* nodes, const int32_t
     std::copy(X.merge_off.begin(), X.merge_off.end(), w + S.off_merge_off);
     std::copy(X.merge_slot.begin(), X.merge_slot.end(), w + S.off_merge_slot);
     std::copy(X.vis.begin(), X.vis.end(), w + S.off_vis);
+    merge_records(X, S.n, w + S.off_merge_rec);
     S.leaf_tail.clear();
     return TP_OK;
 }

@@ -23,6 +23,10 @@ enum UnitKind { KIND_CUDA_CORE = 0, KIND_TENSOR = 1, KIND_TC = 2 };
 // unit words still say KIND_TENSOR).
 constexpr int KIND_PREFILL = 3;
 constexpr int kSchedHeaderWords = 16;
+// Merge record of an occurrence: [slot count, up to 15 slots] (the count is
+// -1 when the occurrence has more slots: the merge then reads the CSR).
+// Fixed-size, so the merge finds it without reading merge_off first.
+constexpr int kMergeRecWords = 16;
 constexpr int32_t kSchedMagic = 0x54505344;
 // Units with fewer query rows may run on the CUDA-core path
 // (TP_DECODE_CUDA_CORE_SMALL); every other unit runs on tensor cores.
@@ -150,6 +154,7 @@ struct DecodeArgs {
 struct MergeArgs {
     const int32_t* merge_off;
     const int32_t* merge_slot;
+    const int32_t* merge_rec;  // [n][kMergeRecWords]
     const float* part_o;
     const float* part_lse;
     uint16_t* out;  // bf16 [n][Hq][hd]
@@ -300,14 +305,14 @@ class BlockPool {
 };
 
 struct Schedule {
-    // header | units | tiles | occ | merge_off | merge_slot, and for a
-    // prefill schedule also unit_pos [n_units] | vis [n]
+    // header | units | tiles | occ | merge_off | merge_slot, for a prefill
+    // schedule also unit_pos [n_units] | vis [n], then merge_rec [n][16]
     std::vector<int32_t> words;
     int32_t n_units = 0, n_tiles = 0, n_occ = 0, n = 0, n_slots = 0, n_merge = 0, n_tensor = 0, n_tc = 0;
     int64_t off_units = 0, off_tiles = 0, off_occ = 0, off_merge_off = 0, off_merge_slot = 0;
     bool prefill = false;
     bool kv_read_once = false;  // see DecodeArgs::kv_read_once
-    int64_t off_unit_pos = 0, off_vis = 0;
+    int64_t off_unit_pos = 0, off_vis = 0, off_merge_rec = 0;
     // (leaf node, word index of the last tile of that leaf) for every place a
     // listed leaf's last block appears: appends that stay inside that block
     // change only these words (see patch_schedule)

@@ -2045,6 +2045,44 @@ __global__ void __launch_bounds__(kTcThreads, 2) decode_tc_kernel(const DecodeAr
 }
 
 // ------------------------------------------------------------------- merge --
+// Fold up to four partial rows (j0 .. j0 + 3 of a chunk of at most 32 slots,
+// rows past cnt masked) into acc; slot and w are the lanes' slot indices and
+// weights (lane k: row k of the chunk). Each row's 128-byte L2 lines are
+// dropped afterwards (a partial row is read by this warp only).
+template <int HD>
+__device__ __forceinline__ void merge_batch(const MergeArgs& a, int qh, int lane, int slot, float w, int j0, int cnt,
+                                            uint64_t pol, float (&acc)[HD / 32]) {
+    constexpr int DPL = HD / 32;
+    constexpr int kLanesPerLine = 128 / (DPL * 4);
+    float wj[4];
+    float x[4][DPL];
+    const float* srcs[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const bool on = j0 + u < cnt;
+        const int64_t sl = __shfl_sync(0xffffffffu, slot, on ? j0 + u : j0);  // off: re-read row j0, weight 0
+        wj[u] = __shfl_sync(0xffffffffu, w, on ? j0 + u : j0) * (on ? 1.f : 0.f);
+        const float* src = a.part_o + (sl * a.hq + qh) * HD + lane * DPL;
+        srcs[u] = on ? src : nullptr;
+        if constexpr (DPL == 4) {
+            const float4 v = ld_f4_hint(src, pol);
+            x[u][0] = v.x, x[u][1] = v.y, x[u][2] = v.z, x[u][3] = v.w;
+        } else {
+            const float2 v = ld_f2_hint(src, pol);
+            x[u][0] = v.x, x[u][1] = v.y;
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) acc[d] += wj[u] * x[u][d];
+    __syncwarp();
+    if ((lane & (kLanesPerLine - 1)) == 0)
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            if (srcs[u]) l2_discard(srcs[u]);
+}
+
 template <int HD>
 __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
     constexpr int DPL = HD / 32;  // dims per lane: 4 or 2
@@ -2053,104 +2091,97 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
     if (blockIdx.x == 0 && threadIdx.x < 3) a.counters[threadIdx.x] = 0;  // decode is done: re-arm its counters
     if (warp_global >= a.n * a.hq) return;
     const int i = warp_global / a.hq, qh = warp_global % a.hq;
-    const int beg = a.merge_off[i], ns = a.merge_off[i + 1] - beg;
-    if (!check(merge_range_ok(beg, beg + ns, a.n_merge) && (ns == 0 || a.n_slots > 0), a.err)) return;
-    if (ns == 0) return;  // written directly by its only unit
     float acc[DPL];
 #pragma unroll
     for (int d = 0; d < DPL; ++d) acc[d] = 0.f;
     float M = -INFINITY, L = 0.f;
     const uint64_t pol = l2_evict_first();  // each partial row is read once
-    // slots in chunks of 32: lane k fetches slot k's index and LSE, then the
-    // warp folds the chunk's partial rows, four loads in flight per lane
-    for (int c0 = 0; c0 < ns; c0 += 32) {
-        const int k = c0 + lane;
-        int slot = 0;
-        float lse = -INFINITY;
-        if (k < ns) {
-            slot = a.merge_slot[beg + k];
-            if (check(in_range(slot, a.n_slots), a.err))
-                lse = a.part_lse[(int64_t)slot * a.hq + qh];
-            else
-                slot = 0;  // weight 0, a valid row to read
+    // The occurrence's merge record, in one round trip: lane k < 16 holds
+    // word k ([count, slots...]).
+    const int rw = lane < kMergeRecWords ? a.merge_rec[(int64_t)i * kMergeRecWords + lane] : 0;
+    const int ns_rec = __shfl_sync(0xffffffffu, rw, 0);
+    if (ns_rec >= 0) {
+        // up to 15 slots: lane k takes slot k; its LSE and the first four
+        // partial rows are loaded together, then folded
+        const int ns = ns_rec;
+        if (!check(ns < kMergeRecWords, a.err) || ns == 0) return;  // 0: written directly by its only unit
+        int slot = __shfl_sync(0xffffffffu, rw, (lane + 1) & 31);  // every lane shuffles
+        const int first = __shfl_sync(0xffffffffu, rw, 1);
+        if (lane >= ns)
+            slot = first;  // a valid row (weight 0)
+        else if (!check(in_range(slot, a.n_slots), a.err))
+            slot = 0;
+        float x0[4][DPL];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int64_t sl = __shfl_sync(0xffffffffu, slot, u < ns ? u : 0);
+            const float* src = a.part_o + (sl * a.hq + qh) * HD + lane * DPL;
+            if constexpr (DPL == 4) {
+                const float4 v = ld_f4_hint(src, pol);
+                x0[u][0] = v.x, x0[u][1] = v.y, x0[u][2] = v.z, x0[u][3] = v.w;
+            } else {
+                const float2 v = ld_f2_hint(src, pol);
+                x0[u][0] = v.x, x0[u][1] = v.y;
+            }
         }
-        float cm = lse;
+        const float lse = lane < ns ? a.part_lse[(int64_t)slot * a.hq + qh] : -INFINITY;
+        M = lse;
 #pragma unroll
-        for (int off = 16; off; off >>= 1) cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, off));
-        const float m_new = fmaxf(M, cm);
-        const float keep = (M == -INFINITY) ? 0.f : fast_exp2(M - m_new);
+        for (int off = 16; off; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+        const float w = lane < ns ? fast_exp2(lse - M) : 0.f;
+        L = w;
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) acc[d] *= keep;
-        L *= keep;
-        M = m_new;
-        const float w = (k < ns) ? fast_exp2(lse - M) : 0.f;
-        float ws = w;
+        for (int off = 16; off; off >>= 1) L += __shfl_xor_sync(0xffffffffu, L, off);
 #pragma unroll
-        for (int off = 16; off; off >>= 1) ws += __shfl_xor_sync(0xffffffffu, ws, off);
-        L += ws;
-        const int cnt = min(32, ns - c0);
-        // A partial row is read by this warp only (slots are per leaf
-        // occurrence): once folded, its lines are dropped from L2 instead of
-        // being written back to HBM. Each 128-byte line is dropped by the
-        // first lane that read from it, after the warp has used the loads.
-        constexpr int kLanesPerLine = 128 / (DPL * 4);
-        const bool line_lead = (lane & (kLanesPerLine - 1)) == 0;
-        int j = 0;
-        for (; j + 4 <= cnt; j += 4) {
-            float wj[4];
-            float x[4][DPL];
-            const float* srcs[4];
+        for (int u = 0; u < 4; ++u) {
+            const float wu = __shfl_sync(0xffffffffu, w, u) * (u < ns ? 1.f : 0.f);
+#pragma unroll
+            for (int d = 0; d < DPL; ++d) acc[d] += wu * x0[u][d];
+        }
+        {
+            constexpr int kLanesPerLine = 128 / (DPL * 4);
+            __syncwarp();
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
-                const int64_t sl = __shfl_sync(0xffffffffu, slot, j + u);
-                wj[u] = __shfl_sync(0xffffffffu, w, j + u);
-                const float* src = a.part_o + (sl * a.hq + qh) * HD + lane * DPL;
-                srcs[u] = src;
-                if constexpr (DPL == 4) {
-                    const float4 v = ld_f4_hint(src, pol);
-                    x[u][0] = v.x, x[u][1] = v.y, x[u][2] = v.z, x[u][3] = v.w;
-                } else {
-                    const float2 v = ld_f2_hint(src, pol);
-                    x[u][0] = v.x, x[u][1] = v.y;
-                }
+                const int64_t sl = __shfl_sync(0xffffffffu, slot, u < ns ? u : 0);  // every lane shuffles
+                if (u < ns && (lane & (kLanesPerLine - 1)) == 0) l2_discard(a.part_o + (sl * a.hq + qh) * HD + lane * DPL);
             }
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-#pragma unroll
-                for (int d = 0; d < DPL; ++d) acc[d] += wj[u] * x[u][d];
-            __syncwarp();
-            if (line_lead)
-#pragma unroll
-                for (int u = 0; u < 4; ++u) l2_discard(srcs[u]);
         }
-        if (j < cnt) {  // the last 1-3 rows as one batch, all loads in flight together
-            float wj[4];
-            float x[4][DPL];
-            const float* srcs[4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const bool on = j + u < cnt;
-                const int64_t sl = __shfl_sync(0xffffffffu, slot, on ? j + u : j);  // off: re-read row j, weight 0
-                wj[u] = __shfl_sync(0xffffffffu, w, on ? j + u : j) * (on ? 1.f : 0.f);
-                const float* src = a.part_o + (sl * a.hq + qh) * HD + lane * DPL;
-                srcs[u] = on ? src : nullptr;
-                if constexpr (DPL == 4) {
-                    const float4 v = ld_f4_hint(src, pol);
-                    x[u][0] = v.x, x[u][1] = v.y, x[u][2] = v.z, x[u][3] = v.w;
-                } else {
-                    const float2 v = ld_f2_hint(src, pol);
-                    x[u][0] = v.x, x[u][1] = v.y;
-                }
+        for (int j = 4; j < ns; j += 4) merge_batch<HD>(a, qh, lane, slot, w, j, ns, pol, acc);
+    } else {
+        // more slots: the CSR, in chunks of 32 -- lane k fetches slot k's
+        // index and LSE, then the warp folds the chunk's partial rows, four
+        // loads in flight per lane
+        const int beg = a.merge_off[i], ns = a.merge_off[i + 1] - beg;
+        if (!check(merge_range_ok(beg, beg + ns, a.n_merge) && (ns == 0 || a.n_slots > 0), a.err)) return;
+        if (ns == 0) return;
+        for (int c0 = 0; c0 < ns; c0 += 32) {
+            const int k = c0 + lane;
+            int slot = 0;
+            float lse = -INFINITY;
+            if (k < ns) {
+                slot = a.merge_slot[beg + k];
+                if (check(in_range(slot, a.n_slots), a.err))
+                    lse = a.part_lse[(int64_t)slot * a.hq + qh];
+                else
+                    slot = 0;  // weight 0, a valid row to read
             }
+            float cm = lse;
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
+            for (int off = 16; off; off >>= 1) cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, off));
+            const float m_new = fmaxf(M, cm);
+            const float keep = (M == -INFINITY) ? 0.f : fast_exp2(M - m_new);
 #pragma unroll
-                for (int d = 0; d < DPL; ++d) acc[d] += wj[u] * x[u][d];
-            __syncwarp();
-            if (line_lead)
+            for (int d = 0; d < DPL; ++d) acc[d] *= keep;
+            L *= keep;
+            M = m_new;
+            const float w = (k < ns) ? fast_exp2(lse - M) : 0.f;
+            float ws = w;
 #pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    if (srcs[u]) l2_discard(srcs[u]);
+            for (int off = 16; off; off >>= 1) ws += __shfl_xor_sync(0xffffffffu, ws, off);
+            L += ws;
+            const int cnt = min(32, ns - c0);
+            for (int j = 0; j < cnt; j += 4) merge_batch<HD>(a, qh, lane, slot, w, j, cnt, pol, acc);
         }
     }
     const float inv = 1.f / L;

@@ -130,13 +130,21 @@ def plant(name, w, pool_blocks, hkv):
     if name == "merge_slot_past_partials":
         w[x["off_mslot"] + 7] = x["n_slots"]
         return "merge_slots"
+    off_mrec = x["off_mslot"] + x["n_merge"]
+    if name == "merge_record_count_wrong":
+        w[off_mrec + 16 * 3] += 1
+        return "merge_ranges"
+    if name == "merge_record_slot_past_partials":
+        w[off_mrec + 16 * 5 + 1] = x["n_slots"]
+        return "merge_slots"
     raise ValueError(name)
 
 
 PLANTS = ["tile_block_past_pool", "tile_too_many_tokens", "tile_negative", "unit_tiles_past_section",
           "unit_too_long", "unit_kv_head", "unit_rows_past_kind", "unit_occurrences_past_list",
           "unit_slot_past_partials", "unit_direct_write_in_decode", "unit_kind_out_of_order",
-          "occurrence_past_rows", "merge_range_backwards", "merge_range_past_list", "merge_slot_past_partials"]
+          "occurrence_past_rows", "merge_range_backwards", "merge_range_past_list", "merge_slot_past_partials",
+          "merge_record_count_wrong", "merge_record_slot_past_partials"]
 
 
 @pytest.mark.parametrize("name", PLANTS)

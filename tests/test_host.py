@@ -281,6 +281,21 @@ def _expand(tiles):
     return out
 
 
+def check_merge_records(S):
+    """Each occurrence's fixed-size merge record holds its CSR slots: count,
+    then the slots in order, zero-padded; -1 when it has more than 15."""
+    rec = S["merge_rec"]
+    assert rec.shape == (len(S["merge_off"]) - 1, 16)
+    for i in range(rec.shape[0]):
+        beg, end = int(S["merge_off"][i]), int(S["merge_off"][i + 1])
+        if end - beg >= 16:
+            assert rec[i, 0] == -1 and not rec[i, 1:].any()
+        else:
+            assert rec[i, 0] == end - beg
+            assert rec[i, 1:1 + end - beg].tolist() == S["merge_slot"][beg:end].tolist()
+            assert not rec[i, 1 + end - beg:].any()
+
+
 def check_schedule(f, ids, model, script, leaves_sid, flags=0):
     heads = script.heads
     g = heads.group
@@ -332,6 +347,7 @@ def check_schedule(f, ids, model, script, leaves_sid, flags=0):
             covered[(i, qh)] += tok
             slots_of[(i, qh)].add(sbase + p)
     n = len(leaves)
+    check_merge_records(S)
     for i in range(n):
         want = sorted(model.path_slots(leaves_sid[i]).tolist())
         mslots = S["merge_slot"][S["merge_off"][i]:S["merge_off"][i + 1]].tolist()
