@@ -549,7 +549,8 @@ tp_status tp_debug_gather(tp_tree* tree, tp_node leaf, void* K_out, void* V_out,
  *   [0] magic 0x54505344, [1] n_units, [2] n_tiles, [3] n_occ_entries,
  *   [4] n (leaf occurrences), [5] n_slots, [6] n_merge_entries, [7] group g,
  *   [8] n_mma_units, [9] n_tcgen05_units, [10] 0 (1 for prefill schedules),
- *   [11] 16 (words per merge record), [12..15] reserved (0),
+ *   [11] 16 (words per merge record; 0 in prefill schedules, which have
+ *   none), [12..15] reserved (0),
  *   then units  [n_units][8]: tile_off, n_tiles, occ_off, row0, n_rows,
  *                             slot_base, kv_head, kind (0 CUDA-core,
  *                             1 mma.sync, 2 tcgen05); tcgen05 units first,
@@ -588,9 +589,10 @@ tp_status tp_debug_schedule(tp_tree* tree, const tp_node* leaves, int32_t n, uin
 tp_status tp_debug_check_schedule(tp_tree* tree, const int32_t* words, int64_t n_words, int64_t* violations);
 
 /* The schedule tp_prefill would run, in the layout above with header word
- * [10] = 1 and two more sections before merge_rec: unit_pos [n_units] (path
- * position of each unit's first token) and vis [n] (tokens of its path that
- * occurrence i -- query token i -- may see). Occurrences are the query
+ * [10] = 1, no merge records ([11] = 0) and two more sections in their
+ * place: unit_pos [n_units] (path position of each unit's first token) and
+ * vis [n] (tokens of its path that occurrence i -- query token i -- may
+ * see). Occurrences are the query
  * tokens; units are tcgen05 units (mma.sync units with TP_MMA_SYNC); a unit
  * row whose occurrence sees nothing of the unit is computed but has no merge
  * entry. */

@@ -351,7 +351,8 @@ def _parse_schedule(w: np.ndarray) -> Dict[str, np.ndarray]:
         out["vis"] = w[off + n_units: off + n_units + n]
         off += n_units + n
     rw = int(w[11])
-    out["merge_rec"] = w[off: off + n * rw].reshape(n, rw)
+    if rw:
+        out["merge_rec"] = w[off: off + n * rw].reshape(n, rw)
     return out
 
 

@@ -214,7 +214,8 @@ tp_status ensure_device(tp_tree* t, T*& ptr, int64_t& cap, int64_t need, const c
     return st;
 }
 
-tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O, float* LSE);
+tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O, float* LSE,
+                       const int32_t* d_sched = nullptr);
 
 // What a schedule's words index into (checked by the bounds-checked build).
 tp::Extents extents_of(const tp_tree* t, const tp::Schedule& S) {
@@ -348,11 +349,17 @@ tp_status tp_tree_destroy(tp_tree* t) {
         if (t->h_pinned[k]) cudaFreeHost(t->h_pinned[k]);
         if (t->h_pinned_ev[k]) cudaEventDestroy(t->h_pinned_ev[k]);
     }
-    for (cudaStream_t s : {t->hp_h2d, t->hp_d2h})
+    for (cudaStream_t s : {t->hp_h2d, t->hp_d2h, t->pf_copy})
         if (s) {
             cudaStreamSynchronize(s);
             cudaStreamDestroy(s);
         }
+    for (int k = 0; k < 2; ++k) {
+        for (cudaEvent_t e : {t->pf_up[k], t->pf_done[k]})
+            if (e) cudaEventDestroy(e);
+        if (t->d_pf[k]) cudaFree(t->d_pf[k]);
+        if (t->h_pf[k]) cudaFreeHost(t->h_pf[k]);
+    }
     for (int k = 0; k < 2; ++k) {
         for (cudaEvent_t e : {t->hp_up[k], t->hp_done[k], t->hp_down[k]})
             if (e) cudaEventDestroy(e);
@@ -640,14 +647,51 @@ tp_status tp_prefill(tp_tree* t, const tp_node* nodes, const int32_t* n_queries,
     if (!t->cfg.pool) return fail(t, TP_ERR_INVALID_ARG, "metadata-only tree cannot run attention");
     if (!Q || !O || !LSE || !aligned(Q, 16) || !aligned(O, 16) || !aligned(LSE, 4))
         return fail(t, TP_ERR_INVALID_ARG, "Q/O must be 16-byte and LSE 4-byte aligned device pointers");
-    t->sched_valid = false;  // the cached decode schedule's device copy is overwritten
-    tp::Schedule& S = t->sched;
+    tp::Schedule& S = t->pf_sched;
     tp_status st = tp::build_prefill_schedule(t, nodes, n_queries, n, flags, S);
     if (st != TP_OK) return st;
     if (S.n == 0) return TP_OK;
-    st = upload_schedule(t, S);
+    // device buffer b: uploaded on the copy stream once the kernels of the
+    // call two back (its last reader) are done; the attention waits for it
+    cudaError_t e = cudaSuccess;
+    if (!t->pf_copy) {
+        e = cudaStreamCreateWithFlags(&t->pf_copy, cudaStreamNonBlocking);
+        for (int k = 0; k < 2 && e == cudaSuccess; ++k)
+            for (cudaEvent_t* ev : {&t->pf_up[k], &t->pf_done[k]})
+                if (e == cudaSuccess) e = cudaEventCreateWithFlags(ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) return cuda_fail(t, e, "prefill upload stream");
+    }
+    const int b = (int)(t->pf_calls & 1);
+    const int64_t words = (int64_t)S.words.size();
+    if (t->d_pf_cap[b] < words) {  // grow: the buffer's last reader must be done before it is freed
+        e = cudaEventSynchronize(t->pf_done[b]);
+        if (e != cudaSuccess) return cuda_fail(t, e, "cudaEventSynchronize");
+        st = ensure_device(t, t->d_pf[b], t->d_pf_cap[b], words, "prefill schedule buffer");
+        if (st != TP_OK) return st;
+    }
+    e = cudaEventSynchronize(t->pf_up[b]);  // the pinned buffer's previous upload has left it
+    if (e != cudaSuccess) return cuda_fail(t, e, "cudaEventSynchronize");
+    if (t->h_pf_cap[b] < words) {
+        if (t->h_pf[b]) cudaFreeHost(t->h_pf[b]);
+        t->h_pf[b] = nullptr;
+        t->h_pf_cap[b] = 0;
+        e = cudaHostAlloc((void**)&t->h_pf[b], (size_t)words * 4, cudaHostAllocDefault);
+        if (e != cudaSuccess) return cuda_fail(t, e, "cudaHostAlloc");
+        t->h_pf_cap[b] = words;
+    }
+    std::memcpy(t->h_pf[b], S.words.data(), (size_t)words * 4);
+    e = cudaStreamWaitEvent(t->pf_copy, t->pf_done[b], 0);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(t->d_pf[b], t->h_pf[b], (size_t)words * 4, cudaMemcpyHostToDevice, t->pf_copy);
+    if (e == cudaSuccess) e = cudaEventRecord(t->pf_up[b], t->pf_copy);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(t->stream, t->pf_up[b], 0);
+    if (e != cudaSuccess) return cuda_fail(t, e, "prefill schedule upload");
+    st = run_schedule(t, S, Q, O, LSE, t->d_pf[b]);
     if (st != TP_OK) return st;
-    return run_schedule(t, S, Q, O, LSE);
+    e = cudaEventRecord(t->pf_done[b], t->stream);
+    if (e != cudaSuccess) return cuda_fail(t, e, "cudaEventRecord");
+    ++t->pf_calls;
+    return TP_OK;
 }
 
 }  // extern "C"
@@ -756,8 +800,9 @@ tp_status tp_debug_prefill_schedule(tp_tree* t, const tp_node* nodes, const int3
 
 namespace {
 // Launch the attention and merge kernels of a schedule already on the
-// device (t->d_sched).
-tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O, float* LSE) {
+// device (at d_sched; the decode cache's t->d_sched when null).
+tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O, float* LSE, const int32_t* d_sched) {
+    if (!d_sched) d_sched = t->d_sched;
     const int32_t hq = t->cfg.num_q_heads, hd = t->cfg.head_dim;
     const int64_t part_floats = (int64_t)S.n_slots * hq * (hd + 1);
     tp_status st = ensure_device(t, t->d_part, t->d_part_cap, std::max<int64_t>(part_floats, 1), "partial buffer");
@@ -765,14 +810,14 @@ tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O
 
     tp::DecodeArgs a;
     if (S.prefill) {
-        a.unit_pos = t->d_sched + S.off_unit_pos;
-        a.vis = t->d_sched + S.off_vis;
+        a.unit_pos = d_sched + S.off_unit_pos;
+        a.vis = d_sched + S.off_vis;
         a.out = (uint16_t*)O;
         a.out_lse = LSE;
     }
-    a.units = t->d_sched + S.off_units;
-    a.tiles = t->d_sched + S.off_tiles;
-    a.occ = t->d_sched + S.off_occ;
+    a.units = d_sched + S.off_units;
+    a.tiles = d_sched + S.off_tiles;
+    a.occ = d_sched + S.off_occ;
     a.q = (const uint16_t*)Q;
     a.pool = (const uint8_t*)t->cfg.pool;
     a.part_o = t->d_part;
@@ -807,9 +852,9 @@ tp_status run_schedule(tp_tree* t, const tp::Schedule& S, const void* Q, void* O
     if (e != cudaSuccess) return cuda_fail(t, e, "decode kernel");
 
     tp::MergeArgs m;
-    m.merge_off = t->d_sched + S.off_merge_off;
-    m.merge_slot = t->d_sched + S.off_merge_slot;
-    m.merge_rec = t->d_sched + S.off_merge_rec;
+    m.merge_off = d_sched + S.off_merge_off;
+    m.merge_slot = d_sched + S.off_merge_slot;
+    m.merge_rec = S.off_merge_rec ? d_sched + S.off_merge_rec : nullptr;
     m.part_o = a.part_o;
     m.part_lse = a.part_lse;
     m.out = (uint16_t*)O;
@@ -897,7 +942,7 @@ tp_status tp_decode_noalloc(tp_tree* t, const tp_node* leaves, int32_t n, const 
     tp::MergeArgs m;
     m.merge_off = d_sched + S.off_merge_off;
     m.merge_slot = d_sched + S.off_merge_slot;
-    m.merge_rec = d_sched + S.off_merge_rec;
+    m.merge_rec = S.off_merge_rec ? d_sched + S.off_merge_rec : nullptr;
     m.part_o = a.part_o;
     m.part_lse = a.part_lse;
     m.out = (uint16_t*)O;
@@ -1077,8 +1122,10 @@ tp_status tp_debug_check_schedule(tp_tree* t, const int32_t* w, int64_t n_words,
     const int64_t off_units = tp::kSchedHeaderWords, off_tiles = off_units + (int64_t)n_units * tp::kUnitWords;
     const int64_t off_occ = off_tiles + n_tiles, off_moff = off_occ + n_occ, off_mslot = off_moff + n + 1;
     const int64_t off_mrec = off_mslot + n_merge + (prefill ? (int64_t)n_units + n : 0);
-    if (w[11] != tp::kMergeRecWords) return fail(t, TP_ERR_INVALID_ARG, "bad schedule header (merge records)");
-    const int64_t end = off_mrec + (int64_t)n * tp::kMergeRecWords;
+    const bool has_rec = w[11] == tp::kMergeRecWords;
+    if (w[11] != (prefill ? 0 : tp::kMergeRecWords))
+        return fail(t, TP_ERR_INVALID_ARG, "bad schedule header (merge records)");
+    const int64_t end = off_mrec + (has_rec ? (int64_t)n * tp::kMergeRecWords : 0);
     if (n_words < end) return fail(t, TP_ERR_INVALID_ARG, "schedule shorter than its header says");
     tp::Extents x;
     x.pool_blocks = t->cfg.pool_blocks;
@@ -1103,7 +1150,7 @@ tp_status tp_debug_check_schedule(tp_tree* t, const int32_t* w, int64_t n_words,
     for (int32_t i = 0; i < n; ++i) bad[3] += !tp::merge_range_ok(w[off_moff + i], w[off_moff + i + 1], n_merge);
     for (int64_t k = 0; k < n_merge; ++k) bad[4] += !tp::in_range(w[off_mslot + k], n_slots);
     // merge records: the count of the CSR range (or -1 past 15) and its slots
-    for (int32_t i = 0; i < n; ++i) {
+    for (int32_t i = 0; has_rec && i < n; ++i) {
         const int32_t* r = w + off_mrec + (int64_t)i * tp::kMergeRecWords;
         const int64_t beg = w[off_moff + i], cnt = (int64_t)w[off_moff + i + 1] - beg;
         const bool range_ok = tp::merge_range_ok(w[off_moff + i], w[off_moff + i + 1], n_merge);

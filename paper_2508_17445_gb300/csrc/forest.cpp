@@ -514,8 +514,8 @@ tp_status build_prefill_schedule(tp_tree* t, const tp_node* nodes, const int32_t
     S.off_merge_slot = S.off_merge_off + S.n + 1;
     S.off_unit_pos = S.off_merge_slot + S.n_merge;
     S.off_vis = S.off_unit_pos + S.n_units;
-    S.off_merge_rec = S.off_vis + S.n;
-    const int64_t total = S.off_merge_rec + (int64_t)S.n * kMergeRecWords;
+    S.off_merge_rec = 0;  // no merge records: most query rows are written directly, the rest use the CSR
+    const int64_t total = S.off_vis + S.n;
     if (total >= (int64_t)1 << 31) return fail(t, TP_ERR_INVALID_ARG, "schedule too large");
     S.words.resize((size_t)total);
     int32_t* w = S.words.data();
@@ -531,7 +531,6 @@ tp_status build_prefill_schedule(tp_tree* t, const tp_node* nodes, const int32_t
     w[8] = S.n_tensor;
     w[9] = S.n_tc;
     w[10] = 1;  // prefill schedule
-    w[11] = kMergeRecWords;
     for (int32_t k = 0; k < S.n_units; ++k) {
         std::memcpy(w + S.off_units + (int64_t)k * kUnitWords, &recs[(size_t)k * W], sizeof(int32_t) * kUnitWords);
         w[S.off_unit_pos + k] = recs[(size_t)k * W + kUnitWords];
@@ -541,7 +540,6 @@ tp_status build_prefill_schedule(tp_tree* t, const tp_node* nodes, const int32_t
     std::copy(X.merge_off.begin(), X.merge_off.end(), w + S.off_merge_off);
     std::copy(X.merge_slot.begin(), X.merge_slot.end(), w + S.off_merge_slot);
     std::copy(X.vis.begin(), X.vis.end(), w + S.off_vis);
-    merge_records(X, S.n, w + S.off_merge_rec);
     S.leaf_tail.clear();
     return TP_OK;
 }

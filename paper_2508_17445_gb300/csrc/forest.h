@@ -154,7 +154,7 @@ struct DecodeArgs {
 struct MergeArgs {
     const int32_t* merge_off;
     const int32_t* merge_slot;
-    const int32_t* merge_rec;  // [n][kMergeRecWords]
+    const int32_t* merge_rec;  // [n][kMergeRecWords], or null: the CSR only (prefill schedules)
     const float* part_o;
     const float* part_lse;
     uint16_t* out;  // bf16 [n][Hq][hd]
@@ -305,8 +305,9 @@ class BlockPool {
 };
 
 struct Schedule {
-    // header | units | tiles | occ | merge_off | merge_slot, for a prefill
-    // schedule also unit_pos [n_units] | vis [n], then merge_rec [n][16]
+    // header | units | tiles | occ | merge_off | merge_slot, then for a
+    // decode schedule merge_rec [n][16], for a prefill one unit_pos
+    // [n_units] | vis [n]
     std::vector<int32_t> words;
     int32_t n_units = 0, n_tiles = 0, n_occ = 0, n = 0, n_slots = 0, n_merge = 0, n_tensor = 0, n_tc = 0;
     int64_t off_units = 0, off_tiles = 0, off_occ = 0, off_merge_off = 0, off_merge_slot = 0;
@@ -373,6 +374,21 @@ struct tp_tree {
     int64_t d_gather_cap = 0;
     cudaStream_t side = nullptr;  // second stream for concurrent tcgen05 units
     cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+
+    // prefill schedules (rebuilt every call): two device buffers used in
+    // turn, uploaded on a copy stream of their own once the kernels that read
+    // the buffer two calls back are done, so a call's upload overlaps the
+    // previous call's attention; a host Schedule of their own (the decode
+    // cache keeps its own)
+    tp::Schedule pf_sched;
+    cudaStream_t pf_copy = nullptr;
+    int32_t* d_pf[2] = {nullptr, nullptr};
+    int64_t d_pf_cap[2] = {0, 0};  // words
+    int32_t* h_pf[2] = {nullptr, nullptr};
+    int64_t h_pf_cap[2] = {0, 0};  // words
+    cudaEvent_t pf_up[2] = {nullptr, nullptr};    // buffer's upload landed
+    cudaEvent_t pf_done[2] = {nullptr, nullptr};  // kernels reading the buffer finished
+    uint64_t pf_calls = 0;
 
     // host-buffer calls (tp_decode_host, tp_prefill_host): two staging slots
     // used in turn, uploads and downloads on streams of their own so that a

@@ -2098,8 +2098,8 @@ __global__ void __launch_bounds__(128) merge_kernel(const MergeArgs a) {
     const uint64_t pol = l2_evict_first();  // each partial row is read once
     // The occurrence's merge record, in one round trip: lane k < 16 holds
     // word k ([count, slots...]).
-    const int rw = lane < kMergeRecWords ? a.merge_rec[(int64_t)i * kMergeRecWords + lane] : 0;
-    const int ns_rec = __shfl_sync(0xffffffffu, rw, 0);
+    const int rw = a.merge_rec && lane < kMergeRecWords ? a.merge_rec[(int64_t)i * kMergeRecWords + lane] : -1;
+    const int ns_rec = __shfl_sync(0xffffffffu, rw, 0);  // -1: the CSR (more than 15 slots, or no records)
     if (ns_rec >= 0) {
         // up to 15 slots: lane k takes slot k; its LSE and the first four
         // partial rows are loaded together, then folded
