@@ -59,6 +59,8 @@ def parse():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--flags", type=int, default=0, help="tp_decode_ex flags for the timed steps")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-others", action="store_true",
+                   help="skip the short measurements of the other workloads that follow the default line")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU-baseline work budget")
     return p.parse_args()
 
@@ -527,6 +529,32 @@ def rollout_cpu_baseline(prompts, sh, args, heads, budget_s):
                       f"{tokens} generated tokens; single thread"}
 
 
+PREFILL_SHAPE = (16, 1024, 512)  # leaves per prompt, prompt tokens, segment tokens (all queries)
+
+
+def prefill_setup(seed, n_prompts):
+    """The segment-prefill forest on cuda:0, its query tensors and its flops."""
+    import torch
+
+    import paper_2508_17445_gb300 as tp
+    import workloads
+    fan, plen, seg = PREFILL_SHAPE
+    script = workloads.segment_prefill(seed=seed, n_prompts=n_prompts, prompt_len=plen, fanout=fan, seg_len=seg)
+    h = script.heads
+    forest = tp.Forest(h.num_q_heads, h.num_kv_heads, h.head_dim, pool_blocks=script.upper_bound_blocks(32) + 64,
+                       device="cuda:0")
+    ids = forest.replay(script.ops, kv_fn=lambda i: script.kv(i, "cuda:0"))
+    nodes = [ids[x] for x in script.leaves]
+    counts = [seg] * len(nodes)
+    total = sum(counts)
+    g = torch.Generator(device="cpu").manual_seed(seed)
+    Q = torch.randn(total, h.num_q_heads, h.head_dim, generator=g).to(torch.bfloat16).to("cuda:0")
+    O = torch.empty_like(Q)
+    L = torch.empty(total, h.num_q_heads, dtype=torch.float32, device="cuda:0")
+    flops = 4 * h.head_dim * h.num_q_heads * len(nodes) * sum(plen + j + 1 for j in range(seg))
+    return script, forest, nodes, counts, Q, O, L, flops
+
+
 def bench_prefill(args):
     """Causal multi-query attention over tree paths: 64 prompts of 1024
     tokens, each forked into 16 leaves holding a 512-token segment; one step
@@ -538,20 +566,9 @@ def bench_prefill(args):
     from paper_2508_17445_gb300 import build as lib_build
     lib_build.build()
     n_prompts = args.prompts or 64
-    fan, plen, seg = 16, 1024, 512
-    script = workloads.segment_prefill(seed=args.seed, n_prompts=n_prompts, prompt_len=plen, fanout=fan, seg_len=seg)
-    h = script.heads
-    forest = tp.Forest(h.num_q_heads, h.num_kv_heads, h.head_dim, pool_blocks=script.upper_bound_blocks(32) + 64,
-                       device="cuda:0")
-    ids = forest.replay(script.ops, kv_fn=lambda i: script.kv(i, "cuda:0"))
-    nodes = [ids[x] for x in script.leaves]
-    counts = [seg] * len(nodes)
+    fan, plen, seg = PREFILL_SHAPE
+    script, forest, nodes, counts, Q, O, L, flops = prefill_setup(args.seed, n_prompts)
     total = sum(counts)
-    g = torch.Generator(device="cpu").manual_seed(args.seed)
-    Q = torch.randn(total, h.num_q_heads, h.head_dim, generator=g).to(torch.bfloat16).to("cuda:0")
-    O = torch.empty_like(Q)
-    L = torch.empty(total, h.num_q_heads, dtype=torch.float32, device="cuda:0")
-    flops = 4 * h.head_dim * h.num_q_heads * len(nodes) * sum(plen + j + 1 for j in range(seg))
     for _ in range(args.warmup):
         tp.tp_prefill(forest.handle, nodes, counts, Q, O, L, args.flags)
     torch.cuda.synchronize()
@@ -742,6 +759,89 @@ def bench_advantage(args):
 # --------------------------------------------------------------------------
 # the GPU arm
 # --------------------------------------------------------------------------
+OTHER_DECODE = ("tiny", "qwen7b", "wide_prefix", "no_sharing")
+
+
+def other_workloads(dev, steps, warmup):
+    """Short measurements of the other workloads, after the default line's
+    and on the same GPU, so that one run records every configuration: each
+    other decode forest (leaf-queries/s over `steps` calls timed like the
+    default line's, its attention kernels' and whole call's fractions of the
+    measured copy peak, the no-share speedup) and the prefill path at full
+    size (query tokens/s; TFLOP/s of its attention kernels). Clocks are
+    sampled for the default line only."""
+    import torch
+
+    import paper_2508_17445_gb300 as tp
+    import workloads
+    peak, _ = peaks()
+    stream = torch.cuda.current_stream()
+
+    def timed(fn):
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b)
+
+    out = {"note": f"each: {warmup} warm-up calls, then {steps} timed calls (CUDA events); attention kernel times "
+                   "from a second run of the same calls with event brackets"}
+    for name in OTHER_DECODE:
+        script = workloads.by_name(name, seed=0)
+        desc = describe(script)
+        h = script.heads
+        forest = tp.Forest(h.num_q_heads, h.num_kv_heads, h.head_dim,
+                           pool_blocks=script.upper_bound_blocks(32) + 64, device=dev)
+        ids = forest.replay(script.ops, kv_fn=lambda i, s=script: s.kv(i, dev))
+        leaves = [ids[x] for x in script.leaves]
+        Q = script.q(dev)
+        O = torch.empty((len(leaves), h.num_q_heads, h.head_dim), dtype=torch.bfloat16, device=dev)
+        L = torch.empty((len(leaves), h.num_q_heads), dtype=torch.float32, device=dev)
+
+        def run(k, flags=0):
+            for _ in range(k):
+                tp.tp_decode_ex(forest.handle, leaves, Q, O, L, flags)
+        run(warmup)
+        ms = timed(lambda: run(steps)) / steps
+        tp.tp_profile_start(forest.handle)
+        timed(lambda: run(steps))
+        kt = tp.tp_profile_stop(forest.handle)
+        run(2, tp.TP_DECODE_NO_SHARE)
+        ms_noshare = timed(lambda: run(steps, tp.TP_DECODE_NO_SHARE)) / steps
+        forest.sync()
+        forest.close()
+        algo = desc["unique_kv_bytes"] + desc["q_bytes"]
+        call = algo + desc["o_bytes"] + desc["lse_bytes"]
+        dec_ms = kt["decode"]["ms"] / steps
+        out[name] = {"value": len(leaves) / (ms / 1e3), "unit": UNIT, "ms_per_step": ms,
+                     "attention_frac_of_hbm": algo / (dec_ms / 1e3) / 1e9 / peak,
+                     "call_frac_of_hbm": call / (ms / 1e3) / 1e9 / peak,
+                     "sharing_speedup": ms_noshare / ms, "workload": workload_label(script)}
+        del Q, O, L
+        torch.cuda.empty_cache()
+    script, forest, nodes, counts, Q, O, L, flops = prefill_setup(0, 64)
+    for _ in range(warmup):
+        tp.tp_prefill(forest.handle, nodes, counts, Q, O, L, 0)
+    k = max(1, min(steps, 5))
+    ms = timed(lambda: [tp.tp_prefill(forest.handle, nodes, counts, Q, O, L, 0) for _ in range(k)]) / k
+    tp.tp_profile_start(forest.handle)
+    timed(lambda: [tp.tp_prefill(forest.handle, nodes, counts, Q, O, L, 0) for _ in range(k)])
+    kt = tp.tp_profile_stop(forest.handle)
+    forest.sync()
+    forest.close()
+    att_ms = kt["decode"]["ms"] / k
+    out["prefill"] = {"value": sum(counts) / (ms / 1e3), "unit": "query-tokens/s", "ms_per_step": ms,
+                      "attention_tflops": flops / (att_ms / 1e3) / 1e12,
+                      "frac_of_sustained_bf16": flops / (att_ms / 1e3) / 1e12 / peaks("bf16_tflops_sustained")[0],
+                      "workload": "segment_prefill: 64 prompts of 1024 tokens x 16 leaves, 512-token segments as "
+                                  "causal queries"}
+    del Q, O, L
+    torch.cuda.empty_cache()
+    return out
+
+
 def main():
     args = parse()
     rank = int(os.environ.get("RANK", "0"))
@@ -904,8 +1004,14 @@ def main():
             cb = oracle_rate(script, dev, args.cpu_seconds)
             line["cpu_baseline"] = {k: cb[k] for k in ("value", "unit", "cores", "kind", "sample", "value_one_core",
                                                        "one_core_sample")}
-        print(json.dumps(line), flush=True)
     forest.close()
+    if rank == 0:
+        if (world == 1 and not args.no_others and args.workload == DEFAULT_WORKLOAD and args.prompts is None
+                and args.flags == 0):
+            del Q, O, LSE
+            torch.cuda.empty_cache()
+            line["other_workloads"] = other_workloads(dev, min(args.steps, 10), max(args.warmup, 3))
+        print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
 
