@@ -736,12 +736,14 @@ def bench_advantage(args):
         "config": {"workload": f"output trees of a {n_prompts}-prompt rollout batch (w=16, 14 x 512): "
                                f"{len(leaves)} trajectories, {n_nodes} nodes, mean depth {depth:.1f}"},
         "roofline": {"bound": "hbm", "achieved": algo / (ms / 1e3) / 1e9, "peak": peak, "unit": "GB/s",
-                     "frac": algo / (ms / 1e3) / 1e9 / peak, "traffic": None, "kernel": "advantage_kernel",
-                     "note": "one CTA; a few hundred KB per call: launch- and latency-bound, not bandwidth-bound",
+                     "frac": algo / (ms / 1e3) / 1e9 / peak, "traffic": None,
+                     "kernel": "advantage_{init,walk,means,abar}_kernel",
+                     "note": "four small launches (fp64 sub-group sums, means, pooled A_i, normalisation); a few "
+                             "hundred KB per call: launch- and latency-bound, not bandwidth-bound",
                      "peak_source": f"{kind} hbm_gbs"},
         "e2e": {"value": len(leaves) / e2e_s, "unit": "trajectories/s", "h2d_bytes_per_step": 8 * len(leaves),
                 "d2h_bytes_per_step": 4 * len(leaves)},
-        "gpu_launches": args.steps, "clocks": clocks,
+        "gpu_launches": 4 * args.steps, "clocks": clocks,
     }
     if not args.no_cpu_baseline:
         import oracle.advantage as OA

@@ -519,7 +519,9 @@ tp_status tp_synth_tokens(tp_tree* tree, uint64_t seed, tp_node node, int32_t po
  * parent table was malformed (an id out of range or a cycle; the affected
  * trajectories are rejected). workspace: device, 8-byte aligned, at least
  * tp_advantage_workspace_bytes(n_nodes, n_out) bytes. Fp64 accumulation,
- * one CTA, asynchronous on cuda_stream. Errors (tp_last_error(NULL)):
+ * four kernels (clear, ancestor sums, sub-group means, per-trajectory A_i
+ * with the last CTA normalising), asynchronous on cuda_stream; calls
+ * sharing a workspace must not overlap. Errors (tp_last_error(NULL)):
  * TP_ERR_INVALID_ARG, TP_ERR_CUDA.
  */
 int64_t tp_advantage_workspace_bytes(int32_t n_nodes, int32_t n_out);

@@ -400,107 +400,175 @@ __global__ void rollout_step_kernel(const StepArgs a) {
 }
 
 // -------------------------------------------------------- tree advantage --
-// Eq. tree_ae over a node table, in one CTA (the tables are small: a few
-// thousand trajectories of a rollout batch). Phases, separated by barriers:
-//   1. every output adds its reward to each strict ancestor's (count, sum)
-//      and folds it into its root's reward range;
-//   2. A_i = mean over those ancestors x of (R_i - sum_x / count_x), for
-//      outputs whose query's rewards are not all equal;
-//   3. mean and (population) std of the A_i over the accepted outputs;
-//   4. adv_i = A_i / std (0 for rejected outputs, or when std is 0).
-constexpr int kAdvThreads = 1024;
+// Eq. tree_ae over a node table, in fp64 and in four launches spread over
+// the SMs (GB300 runs fp64 at a small fraction of its fp32 rate per SM, so
+// one CTA doing every output's divisions was fp64-bound):
+//   init   every node's (count, sum) and reward range cleared;
+//   walk   every output adds its reward to each strict ancestor's (count,
+//          sum) and folds it into its root's reward range;
+//   means  every node's sum_x / count_x, once (fp64 divisions are slow,
+//          and the ancestors of many outputs coincide);
+//   abar   A_i = mean over those ancestors x of (R_i - sum_x / count_x), for
+//          outputs whose query's rewards are not all equal, with the sums of
+//          A_i and of accepted outputs; the last CTA to finish takes the mean
+//          and (population) std over the accepted outputs and writes
+//          adv_i = A_i / std (0 for rejected outputs, or when std is 0).
+// Workspace: cnt[n] | kmin[n] | kmax[n] | sum[n] (fp64) | abar[n_out] |
+// root[n_out] | depth[n_out] | totals (fp64 s, c) | bad flag | CTA ticket.
+constexpr int kAdvThreads = 256;      // init and the final pass
+constexpr int kAdvWalkThreads = 32;   // one warp per CTA: outputs spread over many SMs
+constexpr int kAdvAbarThreads = 128;  // the last CTA also runs the final pass over every output
+
+struct AdvWs {
+    int32_t* cnt;
+    uint32_t* kmin;
+    uint32_t* kmax;
+    double* sum;
+    double* abar;
+    int32_t* root_of;
+    int32_t* depth_of;
+    double* tot;      // [2]: sum of A_i, accepted outputs
+    int32_t* flags;   // [2]: malformed table, CTAs of the abar launch done
+};
+
+__host__ __device__ __forceinline__ int64_t adv_tail_offset(int64_t n_nodes, int64_t n_out) {
+    return ((12 * n_nodes + 7) / 8) * 8 + 8 * n_nodes + 8 * n_out + 8 * n_out;
+}
+
+__device__ __forceinline__ AdvWs adv_ws(const AdvantageArgs& a) {
+    AdvWs w;
+    w.cnt = reinterpret_cast<int32_t*>(a.ws);
+    w.kmin = reinterpret_cast<uint32_t*>(w.cnt + a.n_nodes);
+    w.kmax = w.kmin + a.n_nodes;
+    w.sum = reinterpret_cast<double*>(a.ws + ((12ll * a.n_nodes + 7) / 8) * 8);
+    w.abar = w.sum + a.n_nodes;
+    w.root_of = reinterpret_cast<int32_t*>(w.abar + a.n_out);
+    w.depth_of = w.root_of + a.n_out;
+    w.tot = reinterpret_cast<double*>(a.ws + adv_tail_offset(a.n_nodes, a.n_out));
+    w.flags = reinterpret_cast<int32_t*>(w.tot + 2);
+    return w;
+}
 
 __device__ __forceinline__ uint32_t reward_key(float r) {  // order-preserving float -> uint
     const uint32_t u = __float_as_uint(r);
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
+template <int THREADS>
 __device__ double block_sum(double v, double* red) {
     for (int off = 16; off; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    if (THREADS == 32) return v;
     __syncthreads();
     if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
     __syncthreads();
     double s = 0.0;
-    for (int k = 0; k < kAdvThreads / 32; ++k) s += red[k];  // same order in every thread
+    for (int k = 0; k < THREADS / 32; ++k) s += red[k];  // same order in every thread
+    __syncthreads();
     return s;
 }
 
-__global__ void __launch_bounds__(kAdvThreads) advantage_kernel(const AdvantageArgs a) {
-    __shared__ double red[kAdvThreads / 32];
-    __shared__ int bad;
-    const int tid = threadIdx.x;
-    int32_t* cnt = reinterpret_cast<int32_t*>(a.ws);
-    uint32_t* kmin = reinterpret_cast<uint32_t*>(cnt + a.n_nodes);
-    uint32_t* kmax = kmin + a.n_nodes;
-    double* sum = reinterpret_cast<double*>(a.ws + ((12ll * a.n_nodes + 7) / 8) * 8);
-    double* abar = sum + a.n_nodes;
-    int32_t* root_of = reinterpret_cast<int32_t*>(abar + a.n_out);
-    int32_t* depth_of = root_of + a.n_out;
-    if (tid == 0) bad = 0;
-    for (int x = tid; x < a.n_nodes; x += kAdvThreads) {
-        cnt[x] = 0;
-        sum[x] = 0.0;
-        kmin[x] = 0xffffffffu;
-        kmax[x] = 0u;
+__global__ void __launch_bounds__(kAdvThreads) advantage_init_kernel(const AdvantageArgs a) {
+    const AdvWs w = adv_ws(a);
+    for (int64_t x = (int64_t)blockIdx.x * kAdvThreads + threadIdx.x; x < a.n_nodes;
+         x += (int64_t)gridDim.x * kAdvThreads) {
+        w.cnt[x] = 0;
+        w.sum[x] = 0.0;
+        w.kmin[x] = 0xffffffffu;
+        w.kmax[x] = 0u;
     }
-    __syncthreads();
-    for (int i = tid; i < a.n_out; i += kAdvThreads) {
-        const int32_t lf = a.leaf[i];
-        root_of[i] = -1;
-        depth_of[i] = 0;
-        if (lf < 0 || lf >= a.n_nodes) {
-            bad = 1;
-            continue;
-        }
-        const float r = a.reward[i];
-        int32_t root = lf, depth = 0;
-        for (int32_t x = a.parent[lf]; x != -1; x = a.parent[x]) {
-            if (x < -1 || x >= a.n_nodes || depth >= a.n_nodes) {  // malformed table: stop
-                bad = 1;
-                root = -1;
-                break;
-            }
-            atomicAdd(&cnt[x], 1);
-            atomicAdd(&sum[x], (double)r);
-            root = x;
-            ++depth;
-        }
-        if (root < 0) continue;
-        atomicMin(&kmin[root], reward_key(r));
-        atomicMax(&kmax[root], reward_key(r));
-        root_of[i] = root;
-        depth_of[i] = depth;
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        w.tot[0] = w.tot[1] = 0.0;
+        w.flags[0] = w.flags[1] = 0;
     }
-    __syncthreads();
+}
+
+__global__ void __launch_bounds__(kAdvWalkThreads) advantage_walk_kernel(const AdvantageArgs a) {
+    const AdvWs w = adv_ws(a);
+    const int i = blockIdx.x * kAdvWalkThreads + threadIdx.x;
+    if (i >= a.n_out) return;
+    const int32_t lf = a.leaf[i];
+    w.root_of[i] = -1;
+    w.depth_of[i] = 0;
+    if (lf < 0 || lf >= a.n_nodes) {
+        w.flags[0] = 1;
+        return;
+    }
+    const float r = a.reward[i];
+    int32_t root = lf, depth = 0;
+    for (int32_t x = a.parent[lf]; x != -1; x = a.parent[x]) {
+        if (x < -1 || x >= a.n_nodes || depth >= a.n_nodes) {  // malformed table: stop
+            w.flags[0] = 1;
+            return;
+        }
+        atomicAdd(&w.cnt[x], 1);
+        atomicAdd(&w.sum[x], (double)r);
+        root = x;
+        ++depth;
+    }
+    atomicMin(&w.kmin[root], reward_key(r));
+    atomicMax(&w.kmax[root], reward_key(r));
+    w.root_of[i] = root;
+    w.depth_of[i] = depth;
+}
+
+__global__ void __launch_bounds__(kAdvThreads) advantage_means_kernel(const AdvantageArgs a) {
+    const AdvWs w = adv_ws(a);
+    for (int64_t x = (int64_t)blockIdx.x * kAdvThreads + threadIdx.x; x < a.n_nodes;
+         x += (int64_t)gridDim.x * kAdvThreads)
+        if (w.cnt[x] > 0) w.sum[x] /= (double)w.cnt[x];  // the sub-group mean of G_x
+}
+
+__global__ void __launch_bounds__(kAdvAbarThreads) advantage_abar_kernel(const AdvantageArgs a) {
+    __shared__ double red[kAdvAbarThreads / 32];
+    __shared__ bool last;
+    const AdvWs w = adv_ws(a);
+    const int i = blockIdx.x * kAdvAbarThreads + threadIdx.x;
     double s = 0.0, c = 0.0;
-    for (int i = tid; i < a.n_out; i += kAdvThreads) {
-        const int32_t root = root_of[i], depth = depth_of[i];
-        if (root < 0 || depth == 0 || kmin[root] == kmax[root]) {
-            abar[i] = 0.0;
-            depth_of[i] = 0;  // rejected
-            continue;
+    if (i < a.n_out) {
+        const int32_t root = w.root_of[i], depth = w.depth_of[i];
+        if (root < 0 || depth == 0 || w.kmin[root] == w.kmax[root]) {
+            w.abar[i] = 0.0;
+            w.depth_of[i] = 0;  // rejected
+        } else {
+            const double r = (double)a.reward[i];
+            double acc = 0.0;
+            for (int32_t x = a.parent[a.leaf[i]]; x != -1; x = a.parent[x]) acc += r - w.sum[x];  // sum = mean here
+            s = acc / (double)depth;
+            c = 1.0;
+            w.abar[i] = s;
         }
-        const double r = (double)a.reward[i];
-        double acc = 0.0;
-        for (int32_t x = a.parent[a.leaf[i]]; x != -1; x = a.parent[x]) acc += r - sum[x] / (double)cnt[x];
-        abar[i] = acc / (double)depth;
-        s += abar[i];
-        c += 1.0;
     }
-    const double n_acc = block_sum(c, red);
-    const double mean = n_acc > 0.0 ? block_sum(s, red) / n_acc : 0.0;
+    __threadfence();  // every thread's A_i (and rejections) before the CTA's ticket
+    s = block_sum<kAdvAbarThreads>(s, red);
+    c = block_sum<kAdvAbarThreads>(c, red);
+    if (threadIdx.x == 0) {
+        atomicAdd(&w.tot[0], s);
+        atomicAdd(&w.tot[1], c);
+        __threadfence();  // the totals before the ticket
+        last = atomicAdd(&w.flags[1], 1) == (int)gridDim.x - 1;
+    }
+    __syncthreads();
+    if (!last) return;
+    // the last CTA: mean, std and the normalised advantages of every output
+    // (the other CTAs' writes read through L2, past this SM's L1)
+    __threadfence();
+    const double n_acc = __ldcg(&w.tot[1]);
+    const double mean = n_acc > 0.0 ? __ldcg(&w.tot[0]) / n_acc : 0.0;
     double v = 0.0;
-    for (int i = tid; i < a.n_out; i += kAdvThreads)
-        if (depth_of[i] > 0) v += (abar[i] - mean) * (abar[i] - mean);
-    const double var = n_acc > 0.0 ? block_sum(v, red) / n_acc : 0.0;
-    const double sd = sqrt(var);
-    for (int i = tid; i < a.n_out; i += kAdvThreads)
-        a.adv[i] = (depth_of[i] > 0 && sd > 0.0) ? (float)(abar[i] / sd) : 0.f;
-    if (tid == 0 && a.stats) {
+    for (int k = threadIdx.x; k < a.n_out; k += kAdvAbarThreads)
+        if (__ldcg(&w.depth_of[k]) > 0) {
+            const double d = __ldcg(&w.abar[k]) - mean;
+            v += d * d;
+        }
+    const double var = n_acc > 0.0 ? block_sum<kAdvAbarThreads>(v, red) / n_acc : 0.0;
+    const double sd = sqrt(var), inv_sd = sd > 0.0 ? 1.0 / sd : 0.0;
+    for (int k = threadIdx.x; k < a.n_out; k += kAdvAbarThreads)
+        a.adv[k] = (__ldcg(&w.depth_of[k]) > 0 && sd > 0.0) ? (float)(__ldcg(&w.abar[k]) * inv_sd) : 0.f;
+    if (threadIdx.x == 0 && a.stats) {
         a.stats[0] = n_acc;
         a.stats[1] = mean;
         a.stats[2] = sd;
-        a.stats[3] = bad ? 1.0 : 0.0;
+        a.stats[3] = __ldcg(&w.flags[0]) ? 1.0 : 0.0;
     }
 }
 
@@ -2381,11 +2449,20 @@ cudaError_t launch_synth(const SynthArgs& a, cudaStream_t s) {
 }
 
 int64_t advantage_ws_bytes(int64_t n_nodes, int64_t n_out) {
-    return ((12 * n_nodes + 7) / 8) * 8 + 8 * n_nodes + 8 * n_out + 8 * n_out;
+    return adv_tail_offset(n_nodes, n_out) + 2 * 8 + 2 * 4;
 }
 
 cudaError_t launch_advantage(const AdvantageArgs& a, cudaStream_t s) {
-    advantage_kernel<<<1, kAdvThreads, 0, s>>>(a);
+    const int init_grid = (int)std::min<int64_t>(std::max<int64_t>(1, (a.n_nodes + kAdvThreads - 1) / kAdvThreads),
+                                                 152 * 8);
+    advantage_init_kernel<<<init_grid, kAdvThreads, 0, s>>>(a);
+    const int out_grid = (int)std::max<int64_t>(1, ((int64_t)a.n_out + kAdvWalkThreads - 1) / kAdvWalkThreads);
+    if (a.n_out > 0) {
+        advantage_walk_kernel<<<out_grid, kAdvWalkThreads, 0, s>>>(a);
+        advantage_means_kernel<<<init_grid, kAdvThreads, 0, s>>>(a);
+    }
+    const int abar_grid = (int)std::max<int64_t>(1, ((int64_t)a.n_out + kAdvAbarThreads - 1) / kAdvAbarThreads);
+    advantage_abar_kernel<<<abar_grid, kAdvAbarThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 

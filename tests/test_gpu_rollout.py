@@ -231,7 +231,9 @@ def random_forest(rng, n_roots, n_nodes):
     return out, leaves
 
 
-@pytest.mark.parametrize("seed,n_roots,n_nodes", [(0, 1, 30), (1, 4, 200), (2, 64, 3000), (3, 512, 40000)])
+# 14336 nodes: the largest table kept in shared memory; 14337: the workspace path
+@pytest.mark.parametrize("seed,n_roots,n_nodes", [(0, 1, 30), (1, 4, 200), (2, 64, 3000), (3, 512, 40000),
+                                                  (4, 16, 14336), (5, 16, 14337)])
 def test_advantage_random_forests(seed, n_roots, n_nodes):
     rng = np.random.default_rng(seed)
     parent, leaves = random_forest(rng, n_roots, n_nodes)
