@@ -231,7 +231,7 @@ def random_forest(rng, n_roots, n_nodes):
     return out, leaves
 
 
-# 14336 nodes: the largest table kept in shared memory; 14337: the workspace path
+# (the last two: tables of about 14k nodes, as in a paper-shaped rollout batch)
 @pytest.mark.parametrize("seed,n_roots,n_nodes", [(0, 1, 30), (1, 4, 200), (2, 64, 3000), (3, 512, 40000),
                                                   (4, 16, 14336), (5, 16, 14337)])
 def test_advantage_random_forests(seed, n_roots, n_nodes):
