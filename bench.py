@@ -1012,7 +1012,10 @@ def main():
                 and args.flags == 0):
             del Q, O, LSE
             torch.cuda.empty_cache()
-            line["other_workloads"] = other_workloads(dev, min(args.steps, 10), max(args.warmup, 3))
+            try:  # extra records: a failure here must not cost the default line
+                line["other_workloads"] = other_workloads(dev, min(args.steps, 10), max(args.warmup, 3))
+            except Exception as e:  # noqa: BLE001
+                line["other_workloads"] = {"error": f"{type(e).__name__}: {e}"[:300]}
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
